@@ -1,0 +1,149 @@
+"""Synthetic workloads: parameter-shape lists and seeded input generators.
+
+This module holds no optimiser arithmetic.  It is the one place both the
+CUDA path (tests, benchmark) and the CPU oracle (tests) take their inputs
+from, so the two always see identical values.
+
+Shapes follow PyTorch's ``nn.Linear`` storage, ``[out_features,
+in_features]`` = ``(rows, cols)``.  A shape ``(L, 0)`` is a parameter that is
+not a matrix (bias, LayerNorm scale or shift) with ``L`` elements; the
+optimiser applies the element-wise rule to it.
+
+Query, key and value projections are separate matrices: the paper counts 74
+two-dimensional layers in GPT2-S (Section 4.4), i.e. 12 blocks x {q, k, v,
+o, fc, proj} plus the token and position embeddings.  The token embedding is
+tied to the output head and appears once.
+"""
+import numpy as np
+
+try:  # torch is only needed for the bf16 rounding of gradients
+    import torch
+except ImportError:  # pragma: no cover
+    torch = None
+
+
+def gpt2_shapes(n_layer, n_embd, vocab, ctx, mlp_mult=4, fused_qkv=False):
+    """Parameter shapes of a nanoGPT-style GPT-2 with biases, tied head.
+
+    Returns a list of ``(name, (rows, cols))`` in module order.
+    """
+    d, f = n_embd, mlp_mult * n_embd
+    out = [("wte", (vocab, d)), ("wpe", (ctx, d))]
+    for b in range(n_layer):
+        p = "h%d." % b
+        out += [(p + "ln_1.weight", (d, 0)), (p + "ln_1.bias", (d, 0))]
+        if fused_qkv:
+            out += [(p + "attn.c_attn.weight", (3 * d, d)), (p + "attn.c_attn.bias", (3 * d, 0))]
+        else:
+            for q in ("q", "k", "v"):
+                out += [(p + "attn.%s.weight" % q, (d, d)), (p + "attn.%s.bias" % q, (d, 0))]
+        out += [(p + "attn.c_proj.weight", (d, d)), (p + "attn.c_proj.bias", (d, 0))]
+        out += [(p + "ln_2.weight", (d, 0)), (p + "ln_2.bias", (d, 0))]
+        out += [(p + "mlp.c_fc.weight", (f, d)), (p + "mlp.c_fc.bias", (f, 0))]
+        out += [(p + "mlp.c_proj.weight", (d, f)), (p + "mlp.c_proj.bias", (d, 0))]
+    out += [("ln_f.weight", (d, 0)), ("ln_f.bias", (d, 0))]
+    return out
+
+
+def gpt2_small():
+    """GPT2-S (124M): 12 layers, width 768, vocab 50257, context 1024."""
+    return gpt2_shapes(12, 768, 50257, 1024)
+
+
+def gpt2_nano():
+    """GPT2-Nano-shaped list: 6 layers, width 384, vocab 50304, context 256."""
+    return gpt2_shapes(6, 384, 50304, 256)
+
+
+# Large single matrices of the aspect-ratio sweep (tall, wide, square).
+SWEEP_SHAPES = [(4096, 4096), (4096, 14336), (14336, 4096), (50304, 4096)]
+
+
+def numel(shape):
+    rows, cols = shape
+    return rows if cols == 0 else rows * cols
+
+
+def array_shape(shape):
+    rows, cols = shape
+    return (rows,) if cols == 0 else (rows, cols)
+
+
+def count(shapes):
+    """(N, number of matrices, sum of m + n over matrices, 1-D elements)."""
+    N = mats = mn = one_d = 0
+    for m, n in shapes:
+        if n == 0:
+            one_d += m
+            N += m
+        else:
+            mats += 1
+            mn += m + n
+            N += m * n
+    return N, mats, mn, one_d
+
+
+def bf16_round(a):
+    """Round a float32 array to bf16 (nearest-even) and return the bf16 values as float32."""
+    if torch is None:
+        raise RuntimeError("torch is required for bf16 rounding")
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.to(torch.bfloat16).to(torch.float32).numpy()
+
+
+def normal_list(shapes, seed, std, dtype=np.float32):
+    """One float32 array per shape, i.i.d. N(0, std^2), drawn in list order from ``seed``."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for s in shapes:
+        a = rng.standard_normal(numel(s), dtype=np.float32)
+        a *= np.float32(std)
+        out.append(a.reshape(array_shape(s)).astype(dtype, copy=False))
+    return out
+
+
+class ModelInputs:
+    """Seeded synthetic state for a parameter list.
+
+    ``X`` ~ N(0, x_std^2) float32, ``P`` = 0, and ``grads(step)`` yields
+    float32 arrays ~ N(0, g_std^2), already rounded to bf16 when
+    ``grad_bf16`` (the rounded values are what both sides consume).
+    """
+
+    def __init__(self, shapes, seed, x_std=0.02, g_std=1e-3, grad_bf16=True):
+        self.shapes = list(shapes)
+        self.seed = int(seed)
+        self.g_std = float(g_std)
+        self.grad_bf16 = bool(grad_bf16)
+        self.X = normal_list(self.shapes, [self.seed, 0], x_std)
+        self.P = [np.zeros(array_shape(s), np.float32) for s in self.shapes]
+
+    def grads(self, step):
+        g = normal_list(self.shapes, [self.seed, 1, int(step)], self.g_std)
+        if self.grad_bf16:
+            g = [bf16_round(a) for a in g]
+        return g
+
+
+class QuadraticProblem:
+    """f(X) = 1/2 sum A (.) (X - X*)^2 on an m x n matrix, gradient A (.) (X - X*).
+
+    A ~ U[0.1, 10] and X* ~ N(0, 1), both float32, from ``seed``; X(0) = 0 and
+    P(0) = 0.
+    """
+
+    def __init__(self, m, n, seed):
+        rng = np.random.default_rng(seed)
+        self.A = rng.uniform(0.1, 10.0, size=(m, n)).astype(np.float32)
+        self.Xstar = rng.standard_normal((m, n), dtype=np.float32)
+        self.X0 = np.zeros((m, n), np.float32)
+        self.P0 = np.zeros((m, n), np.float32)
+
+
+def single_matrix_inputs(m, n, seed, steps, x_std=0.02, g_std=0.01):
+    """Single m x n fp32 matrix: X ~ N(0, x_std^2), P = 0, one fresh fp32
+    gradient N(0, g_std^2) per step (all drawn from ``seed``)."""
+    rng = np.random.default_rng(seed)
+    X = (rng.standard_normal((m, n), dtype=np.float32) * np.float32(x_std))
+    G = [(rng.standard_normal((m, n), dtype=np.float32) * np.float32(g_std)) for _ in range(steps)]
+    return X, np.zeros((m, n), np.float32), G
