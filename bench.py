@@ -1,0 +1,450 @@
+#!/usr/bin/env python
+"""Benchmark of the R-iKFAD optimiser step on GB300.
+
+One step = one R-iKFAD update (BACD splitting: kick, drift, symmetric rank-1
+friction, damping) over every tensor of a GPT2-S-shaped parameter set
+(196 tensors, 124,439,808 parameters; fp32 parameters and momenta, bf16
+gradients), i.e. one fused step kernel plus one factor-finalise kernel.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  With N > 1 (launched by torchrun) every rank
+runs its own replica of the step (the update has no exchange step); the
+reported value is the total over ranks divided by the slowest rank's time.
+"""
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import shutil
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "R-iKFAD step Gparams/s and HBM GB/s vs peak, GPT2-S param set, 1 GB300"
+UNIT = "Gparams/s"
+# The paper's GPT2-S R-iKFAD0 hyperparameters (optimised-hyperparameter table).
+HP = dict(alpha=0.0579, mu=1.3637e-6, gamma=0.0, eps_stab=1e-16)
+STEP = 0.0918
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "rikfad_step_kernel__gpt2s.md")
+KERNEL_SOURCES = ["paper_2609_30342_gb300/csrc/rikfad_kernels.cuh",
+                  "paper_2609_30342_gb300/csrc/rikfad_plan.hpp",
+                  "paper_2609_30342_gb300/csrc/rikfad_planner.cpp"]
+
+
+# ------------------------------------------------------------ workloads
+
+def workload(name):
+    from paper_2609_30342_gb300 import workloads as W
+    if name == "gpt2s":
+        named = W.gpt2_small()
+        desc = ("GPT2-S parameter set: 12 layers, width 768, vocab 50257 (tied), ctx 1024, "
+                "separate q/k/v; 74 matrices + 122 vectors")
+        seed = 3
+    elif name == "nano":
+        named = W.gpt2_nano()
+        desc = "GPT2-Nano-shaped parameter set: 6 layers, width 384, vocab 50304, ctx 256"
+        seed = 2
+    elif name.startswith("sweep"):
+        i = int(name[5:] or 0)
+        shp = W.SWEEP_SHAPES[i]
+        named = [("W", shp)]
+        desc = "single %d x %d matrix" % shp
+        seed = 4
+    else:
+        raise SystemExit("unknown workload %r" % name)
+    return named, desc, seed
+
+
+def algorithmic_bytes(shapes, grad_bytes):
+    """Compulsory HBM bytes of one step: every matrix element reads the
+    gradient, X and P and writes X and P (grad + 16 bytes); every vector
+    element also reads and writes its friction (grad + 24 bytes)."""
+    from paper_2609_30342_gb300 import workloads as W
+    N, _, _, one_d = W.count(shapes)
+    return (N - one_d) * (grad_bytes + 16) + one_d * (grad_bytes + 24)
+
+
+# ------------------------------------------------------- distributed glue
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def init_dist(world, backend):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(value, world, device="cpu"):
+    """Maximum of a float over all ranks (identity when world == 1)."""
+    if world == 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(units_per_rank, seconds_max, world):
+    """Whole-job throughput: units processed by all ranks / slowest rank's time."""
+    return units_per_rank * world / seconds_max
+
+
+# ------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id, period_ms=100):
+        self.gpu_id = gpu_id
+        self.period_ms = period_ms
+        self.proc = None
+        self.path = None
+        self.err = None
+
+    def start(self):
+        smi = shutil.which("nvidia-smi")
+        if smi is None:
+            self.err = "nvidia-smi not found"
+            return
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        cmd = [smi, "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+               "-lms", str(self.period_ms)]
+        if self.gpu_id is not None:
+            cmd += ["-i", str(self.gpu_id)]
+        self.out = open(self.path, "w")
+        self.proc = subprocess.Popen(cmd, stdout=self.out, stderr=subprocess.DEVNULL)
+
+    def stop(self):
+        if self.proc is None:
+            return {"unavailable": self.err or "not started"}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        lines = open(self.path).read().strip().splitlines()
+        os.unlink(self.path)
+        sm, mx, pw, reasons = [], [], [], set()
+        for ln in lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+                pw.append(float(f[3]))
+            except ValueError:
+                continue
+            for name, val in zip(self.REASONS, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)),
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": float(max(pw))}
+
+
+# ------------------------------------------------------------ peaks & ncu
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest():
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic():
+    """DRAM bytes per launch of the step kernel from the committed ncu summary,
+    or None if there is none or the kernel changed since it was taken."""
+    try:
+        text = open(PROFILE_SUMMARY).read()
+    except OSError:
+        return None
+    m_sha = re.search(r"kernel_source_digest:\s*([0-9a-f]+)", text)
+    m_b = re.search(r"dram_bytes_per_launch_gpt2s:\s*([0-9.eE+]+)", text)
+    if not (m_sha and m_b) or m_sha.group(1) != kernel_source_digest():
+        return None
+    return float(m_b.group(1))
+
+
+# ------------------------------------------------------------ oracle (CPU)
+
+def oracle_sample(named, seed, budget_s):
+    """Pick the largest sample of the workload that the oracle steps through
+    within budget_s (one step), and the inputs for it."""
+    from paper_2609_30342_gb300 import workloads as W
+    import oracle
+    names = [n for n, _ in named]
+    cands = [("blocks h0-h1", lambda n: n.startswith("h0.") or n.startswith("h1.")),
+             ("block h0", lambda n: n.startswith("h0.")),
+             ("block h0 attention", lambda n: n.startswith("h0.attn.")),
+             ("h0.attn.q", lambda n: n.startswith("h0.attn.q."))]
+    if len(named) == 1:
+        cands = [("whole workload", lambda n: True)]
+    calib = [i for i, n in enumerate(names) if cands[-1][1](n)] or [0]
+    shapes = [named[i][1] for i in calib]
+    inp = W.ModelInputs(shapes, seed=seed)
+    st = oracle.ModelState(shapes, inp.X, inp.P)
+    g = [a.astype(np.float64) for a in inp.grads(0)]
+    t0 = time.perf_counter()
+    st.step(g, STEP, oracle.HParams(**HP))
+    per_param = (time.perf_counter() - t0) / max(W.count(shapes)[0], 1)
+    for label, pred in cands:
+        idx = [i for i, n in enumerate(names) if pred(n)]
+        n_par = W.count([named[i][1] for i in idx])[0]
+        if n_par * per_param <= budget_s or label == cands[-1][0]:
+            return label, idx
+    return cands[-1][0], calib
+
+
+def time_oracle(named, seed, idx, steps, warmup):
+    """Seconds per oracle step over the tensors ``idx`` (float64, 1 thread)."""
+    from paper_2609_30342_gb300 import workloads as W
+    import oracle
+    shapes = [named[i][1] for i in idx]
+    inp = W.ModelInputs(shapes, seed=seed)
+    st = oracle.ModelState(shapes, inp.X, inp.P)
+    g = [a.astype(np.float64) for a in inp.grads(0)]
+    hp = oracle.HParams(**HP)
+    for _ in range(warmup):
+        st.step(g, STEP, hp)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        st.step(g, STEP, hp)
+    return (time.perf_counter() - t0) / steps, W.count(shapes)[0]
+
+
+def cpu_baseline(named, seed, target_s=12.0):
+    label, idx = oracle_sample(named, seed, budget_s=target_s / 3)
+    sec1, n_par = time_oracle(named, seed, idx, 1, 0)
+    reps = int(min(30, max(2, math.ceil(target_s / max(sec1, 1e-6)))))
+    sec, n_par = time_oracle(named, seed, idx, reps, 0)
+    return {"value": n_par / sec / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": "%s of the workload (%d tensors, %d params), %d steps of the float64 C "
+                      "oracle, single thread" % (label, len(idx), n_par, reps)}
+
+
+# ------------------------------------------------------------ our arm
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    from paper_2609_30342_gb300 import rikfad
+    from paper_2609_30342_gb300 import workloads as W
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    init_dist(world, "nccl")
+    rikfad.lib()
+
+    named, desc, seed = workload(args.workload)
+    shapes = [s for _, s in named]
+    N, mats, mn, one_d = W.count(shapes)
+    inp = W.ModelInputs(shapes, seed=seed)
+    grads = inp.grads(0)
+
+    # Gradients live in one flat bf16 buffer (device) with a pinned host twin,
+    # so the end-to-end run copies them in with one transfer per step.
+    offs, total = [], 0
+    for s in shapes:
+        offs.append(total)
+        total += -(-W.numel(s) // 8) * 8
+    g_dev = torch.zeros(max(total, 1), dtype=torch.bfloat16, device=dev)
+    g_host = torch.zeros(max(total, 1), dtype=torch.bfloat16).pin_memory()
+    g_views = []
+    for s, o, a in zip(shapes, offs, grads):
+        n = W.numel(s)
+        g_host[o:o + n].copy_(torch.from_numpy(a.ravel()).to(torch.bfloat16))
+        g_views.append(g_dev[o:o + n].view(W.array_shape(s)))
+    g_dev.copy_(g_host)
+    x = [torch.from_numpy(a).to(dev) for a in inp.X]
+    p = [torch.zeros(W.array_shape(s), dtype=torch.float32, device=dev) for s in shapes]
+    del inp, grads
+
+    opt = rikfad.RIKFAD(shapes, grad_dtype="bf16", **HP)
+    ptrs = opt.pack(x, g_views, p)
+    stream = torch.cuda.current_stream(dev)
+    alg_bytes = algorithmic_bytes(shapes, 2)
+
+    for _ in range(args.warmup):
+        opt.step(STEP, ptrs=ptrs, stream=stream)
+    torch.cuda.synchronize(dev)
+
+    # ---- device-timed region: inputs resident in HBM (2.24 GB > 129 MB L2)
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        uuid = None
+    sampler = ClockSampler(uuid)
+    opt.profile_enable(True)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.25)      # let the sampler take its first reading
+    ev0.record(stream)
+    for _ in range(args.steps):
+        opt.step(STEP, ptrs=ptrs, stream=stream)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = sampler.stop()
+    barrier(world)
+    ms_total = ev0.elapsed_time(ev1)
+    step_ms, fin_ms, nrec = opt.profile_read()
+    opt.profile_enable(False)
+    ms_max = max_over_ranks(ms_total, world, dev)
+    ms_per_step = ms_max / args.steps
+    value = aggregate(N, ms_per_step / 1e3, world) / 1e9
+    kern_ms = step_ms / max(nrec, 1)
+    peak, peak_src = hbm_peak()
+    achieved = alg_bytes / (kern_ms / 1e3) / 1e9
+    traffic = ncu_traffic() if args.workload == "gpt2s" else None
+
+    # ---- end to end: gradients copied in from pinned host memory every step,
+    # the step, and the friction denominators (one float per tensor) read back.
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        g_dev.copy_(g_host, non_blocking=True)
+        opt.step(STEP, ptrs=ptrs, stream=stream)
+        opt.read_denominators(stream)
+    torch.cuda.synchronize(dev)
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
+    barrier(world)
+    e2e = {"value": aggregate(N, e2e_s / args.steps, world) / 1e9, "unit": UNIT,
+           "h2d_bytes_per_step": int(g_host.numel() * g_host.element_size()),
+           "d2h_bytes_per_step": 4 * len(shapes)}
+
+    launches = opt.launches_per_step() * args.steps
+    state = opt.state_bytes(True)
+    full_state = 8 * N
+    opt.close()
+
+    if rank != 0:
+        return None
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded): X ~ N(0, 0.02^2) fp32, P = 0 fp32, grad ~ N(0, 1e-3^2) bf16",
+        "config": {"workload": desc, "params": N, "tensors": len(shapes), "matrices": mats,
+                   "vector_elements": one_d, "grad_dtype": "bf16", "state_dtype": "f32",
+                   "hyperparameters": dict(HP, h=STEP),
+                   "l2": "no flush: %.2f GB of inputs per step > 129 MB L2" % (alg_bytes / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "hbm_gbs_step": round(alg_bytes / (ms_per_step / 1e3) / 1e9, 1),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "kernel": "rikfad_step_kernel", "peak_source": peak_src,
+                     "algorithmic_bytes_per_launch": alg_bytes,
+                     "kernel_ms": round(kern_ms, 5),
+                     "finalize_kernel_ms": round(fin_ms / max(nrec, 1), 5)},
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "state_bytes": {"rikfad": state, "full_friction_ikfad": full_state,
+                        "ratio": round(full_state / state, 3)},
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(named, seed)
+    return line
+
+
+# ------------------------------------------------------------ reference arm
+
+def run_reference(args, rank, world):
+    """The oracle (plain float64 C, one thread) on a bounded sample of the
+    same workload, timed per step on the host cores."""
+    if rank != 0:
+        return None
+    named, desc, seed = workload(args.workload)
+    budget = 150.0 / max(args.steps + args.warmup, 1)
+    label, idx = oracle_sample(named, seed, budget_s=budget)
+    sec, n_par = time_oracle(named, seed, idx, args.steps, args.warmup)
+    value = n_par / sec / 1e9
+    sample = ("%s of the workload (%d tensors, %d params) per step, float64 C oracle, single "
+              "thread" % (label, len(idx), n_par))
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded)", "config": {"workload": desc},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default="gpt2s",
+                    help="gpt2s (default), nano, sweep0..sweep3")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    rank, world, local_rank = dist_env()
+    if world != args.gpus:
+        if world == 1 and args.gpus > 1:
+            raise SystemExit("--gpus %d needs torchrun with %d processes" % (args.gpus, args.gpus))
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line = run_ours(args, rank, world, local_rank)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+        if dist.is_initialized():
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

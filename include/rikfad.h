@@ -1,0 +1,232 @@
+/*
+ * rikfad.h -- C ABI of the GB300 (sm_103a) Rank-1 iKFAD (R-iKFAD) optimiser.
+ *
+ * R-iKFAD ("Low-Rank Friction for Memory-Efficient Transformer Pretraining",
+ * Rajpal & Leimkuhler) is momentum descent with an adaptive friction.  For a
+ * matrix parameter X (m x n) it keeps the full momentum P and two factors
+ * R (m) and C (n) whose outer product gives the friction
+ *     xi~_ij = R_i C_j / (1_m^T R + eps_stab)                       (Eq. xi_def)
+ * (Section 2, Eqs. rikfad_x to rikfad_C).  One optimiser step is the BACD
+ * splitting of Appendix A (Table "Analytical sub-step update rules"):
+ *     B  P^(B) = P_n - h grad f(X_n)
+ *     A  X_{n+1} = X_n + h P^(B)
+ *     C  P^(1) = P^(B) (.) exp(-(h/2) xi~_n)
+ *        R_{n+1} = e^{-alpha h} R_n + (1 - e^{-alpha h})/(mu alpha) [P^(1)]^2 1_n
+ *        C_{n+1} = e^{-alpha h} C_n + (1 - e^{-alpha h})/(mu alpha) ([P^(1)]^2)^T 1_m
+ *        P^(2) = P^(1) (.) exp(-(h/2) xi~_{n+1})
+ *     D  P_{n+1} = P^(2) e^{-gamma h}
+ * Parameters that are not matrices (biases, LayerNorm) follow element-wise
+ * iKFAD (Section 2, "Memory Complexity"): a friction scalar per element
+ * takes the place of xi~ and is filtered from its own [P^(1)]^2.
+ *
+ * Conventions for every call:
+ *   - Pointers named "device" are CUDA device pointers of the device that was
+ *     current when the handle was created; "host" pointers are CPU memory.
+ *   - Tensors are dense and row-major.  A matrix (rows m, cols n) element
+ *     (i, j) is at offset i*n + j.  Parameters and momenta are float32;
+ *     gradients are float32 or bfloat16, fixed per handle.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued on it and nothing waits on the host unless the
+ *     call says so.  The library never synchronises the device.
+ *   - Every call that can fail returns a rikfad_status; on failure
+ *     rikfad_last_error() describes it (thread-local string).  Argument errors
+ *     are detected before any work is enqueued.  Errors of work already
+ *     enqueued surface as RIKFAD_ERR_CUDA on a later call.
+ *   - A handle is not thread-safe: calls on one handle must not overlap.
+ */
+#ifndef RIKFAD_H
+#define RIKFAD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define RIKFAD_API __attribute__((visibility("default")))
+#else
+#define RIKFAD_API
+#endif
+
+/* Status codes. */
+enum rikfad_status {
+    RIKFAD_OK = 0,
+    RIKFAD_ERR_ARG = -1,   /* null pointer, bad shape, bad hyperparameter, bad index */
+    RIKFAD_ERR_ALIGN = -2, /* a pointer does not meet the documented alignment */
+    RIKFAD_ERR_CUDA = -3,  /* a CUDA runtime call or an earlier kernel failed */
+    RIKFAD_ERR_OOM = -4,   /* device or pinned host allocation failed */
+    RIKFAD_ERR_STATE = -6  /* call not valid for this handle (e.g. wrong device) */
+};
+
+/* Gradient element type, fixed per handle. */
+enum rikfad_grad_dtype { RIKFAD_GRAD_F32 = 0, RIKFAD_GRAD_BF16 = 1 };
+
+/* Hyperparameters of Eqs. rikfad_x to rikfad_C and Eq. xi_def: the factor
+ * decay alpha > 0, the friction scale mu > 0, the linear damping gamma >= 0
+ * (gamma = 0 is R-iKFAD0, the paper's default, Section 4.2) and the
+ * stabiliser eps_stab >= 0 (the paper fixes 1e-16, Section 4).  With
+ * eps_stab = 0 the friction is zero while 1^T R = 0 (Theorem 3's convention). */
+typedef struct {
+    double alpha;
+    double mu;
+    double gamma;
+    double eps_stab;
+} rikfad_hparams;
+
+/* Shape of one parameter tensor.  cols >= 1: an m x n matrix (rows = m >= 0)
+ * with factors R (m) and C (n).  cols == 0: a tensor that is not a matrix,
+ * flattened to `rows` >= 0 elements, updated element-wise. */
+typedef struct {
+    int64_t rows;
+    int64_t cols;
+} rikfad_shape;
+
+typedef struct rikfad_handle_s *rikfad_handle;
+
+/*
+ * Create an optimiser for a fixed list of parameter tensors on the current
+ * CUDA device.  Allocates and zeroes the factors R, C and the element-wise
+ * friction (R(0) = C(0) = 0, as in Lemma 1 and the numerical appendix), plus
+ * the reduction workspace, and plans the fused kernels for this list.
+ *   shapes     host array of `ntensors` shapes (ntensors >= 0), copied
+ *   hp         host pointer, copied; alpha, mu > 0, gamma, eps_stab >= 0
+ *   grad_dtype RIKFAD_GRAD_F32 or RIKFAD_GRAD_BF16
+ *   out        receives the handle (NULL on failure)
+ * Errors: RIKFAD_ERR_ARG, RIKFAD_ERR_OOM, RIKFAD_ERR_CUDA.
+ */
+RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
+                             int grad_dtype, rikfad_handle *out);
+
+/* Release the handle and everything it allocated (after a device sync of its
+ * own work).  NULL is accepted. */
+RIKFAD_API void rikfad_destroy(rikfad_handle h);
+
+/*
+ * Enqueue one R-iKFAD step of size `step` (> 0, finite) over every tensor.
+ *   x[t]    device, float32, tensor t's parameters; updated to X_{n+1}
+ *   grad[t] device, float32 or bfloat16 (per handle), grad f(X_n); read only
+ *   p[t]    device, float32, tensor t's momentum in the library's stored form
+ *           (below); updated
+ * The three arrays are host arrays of `ntensors` device pointers, in the
+ * order of the shapes given to rikfad_create; they may change from call to
+ * call (a change costs one small host-to-device copy).  Every pointer must be
+ * 16-byte aligned, except for matrices whose cols is not a multiple of 8 and
+ * for which only natural alignment is required.  Pointers of empty tensors
+ * may be NULL.  x, grad and p must not overlap.
+ *
+ * Stored form of the momentum of a matrix: between steps p holds P^(1) of
+ * the last step (the half-damped momentum) and the library remembers the
+ * pending factor exp(-(h/2) xi~_{n+1}) e^{-gamma h} of sub-steps C and D,
+ * which the next step applies on the fly (the values are identical to the
+ * paper's P_{n+1}).  rikfad_materialize / rikfad_canonical_momentum give the
+ * paper's P_{n+1}.  Element-wise tensors always hold P_{n+1}.  Before the
+ * first step p must hold the initial momentum (normally zeros).
+ */
+RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const void *const *grad,
+                           float *const *p, void *stream);
+
+/*
+ * Turn the stored momenta into the paper's P_{n+1} in place and clear the
+ * pending factor, so the next step starts from canonical momenta.  Use before
+ * checkpointing the momenta or handing them to other code.
+ *   p  host array of ntensors device pointers (same rules as rikfad_step)
+ */
+RIKFAD_API int rikfad_materialize(rikfad_handle h, float *const *p, void *stream);
+
+/*
+ * Write the paper's P_{n+1} of every matrix into `out` without changing the
+ * optimiser's state (the stored momenta and pending factor are left as they
+ * are).  Element-wise tensors are copied.  out[t] must not overlap p[t].
+ */
+RIKFAD_API int rikfad_canonical_momentum(rikfad_handle h, const float *const *p,
+                                         float *const *out, void *stream);
+
+/* Optimiser auxiliary state in bytes, as counted in the paper's memory table
+ * (Appendix "Memory Analysis"): factors R and C of every matrix plus the
+ * element-wise friction (4 bytes each), plus, if include_momentum != 0, the
+ * float32 momentum of every parameter.  Workspace is not included. */
+RIKFAD_API size_t rikfad_state_bytes(rikfad_handle h, int include_momentum);
+
+/* Same count for a shape list, without a handle or a GPU. */
+RIKFAD_API size_t rikfad_state_bytes_for(const rikfad_shape *shapes, int ntensors,
+                                         int include_momentum);
+
+/* Device bytes the handle allocated besides the state (reduction partials,
+ * plan tables, pointer table). */
+RIKFAD_API size_t rikfad_workspace_bytes(rikfad_handle h);
+
+/* The step size whose pending factor the stored momenta still carry (0 after
+ * creation, rikfad_materialize or rikfad_import_state of a materialised
+ * state). */
+RIKFAD_API double rikfad_pending_step(rikfad_handle h);
+
+/*
+ * Copy tensor t's factors to the host (synchronises the device).
+ * Matrix: R_host receives rows floats, C_host cols floats (either may be NULL).
+ * Element-wise tensor: R_host receives its rows friction values; C_host unused.
+ */
+RIKFAD_API int rikfad_get_factors(rikfad_handle h, int t, float *R_host, float *C_host);
+
+/* Overwrite tensor t's factors from the host (same layout as
+ * rikfad_get_factors; values must be finite and >= 0).  Synchronises. */
+RIKFAD_API int rikfad_set_factors(rikfad_handle h, int t, const float *R_host, const float *C_host);
+
+/* Read the friction denominators 1^T R of every matrix (ntensors floats, 0 for
+ * element-wise tensors) into host memory, enqueued on `stream`; the values
+ * are valid once the stream reaches this point (the call itself waits for it). */
+RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *stream);
+
+/*
+ * Checkpoint support.  The state image is rikfad_state_image_bytes(h) bytes:
+ * a 64-byte header (format tag, tensor count, pending step) followed by
+ * every factor and element-wise friction value.  Momenta are not included
+ * (the caller owns them; they are in the stored form of rikfad_step).
+ *   export: dev_dst, device, receives the image (enqueued on stream)
+ *   import: dev_src, device, an image exported by a handle with the same
+ *           shapes and hyperparameters; synchronises to validate the header
+ */
+RIKFAD_API size_t rikfad_state_image_bytes(rikfad_handle h);
+RIKFAD_API int rikfad_export_state(rikfad_handle h, void *dev_dst, void *stream);
+RIKFAD_API int rikfad_import_state(rikfad_handle h, const void *dev_src, void *stream);
+
+/*
+ * Kernel timing.  While enabled, rikfad_step records CUDA events on its
+ * stream around the fused step kernel and around the factor-finalise
+ * kernel.  rikfad_profile_read waits for the recorded events and returns the
+ * summed durations in milliseconds and the number of steps recorded since the
+ * last enable; it then forgets them.
+ */
+RIKFAD_API int rikfad_profile_enable(rikfad_handle h, int enable);
+RIKFAD_API int rikfad_profile_read(rikfad_handle h, double *step_kernel_ms,
+                                   double *finalize_kernel_ms, int64_t *steps);
+
+/* Number of kernel launches one rikfad_step enqueues for this handle. */
+RIKFAD_API int rikfad_launches_per_step(rikfad_handle h);
+
+/*
+ * Work plan for a shape list, computed on the host for `nctas` blocks (no GPU
+ * needed; the same planner rikfad_create uses).  Writes at most `cap` rows of
+ * 8 int64 values into `out` (host) and returns the number of rows the plan
+ * has (so a call with cap = 0 sizes the buffer), or a negative status.  Row:
+ *   { block, tensor, kind (0 matrix rows, 1 element range), col0, width,
+ *     begin, end, slot }
+ * For kind 0 the block updates rows [begin, end) x columns [col0, col0+width)
+ * of the matrix and writes its column partial sums to `slot`; for kind 1 it
+ * updates elements [begin, end).
+ */
+RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, int grad_dtype,
+                                     int nctas, int64_t *out, int64_t cap);
+
+/* Last error message of the calling thread ("" if none). */
+RIKFAD_API const char *rikfad_last_error(void);
+
+/* ABI version of this header: 1. */
+RIKFAD_API int rikfad_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RIKFAD_H */

@@ -73,7 +73,7 @@ def step_matrix(X, P, R, C, G, h, hp):
     m, n = X.shape
     if P.shape != (m, n) or G.shape != (m, n) or R.shape != (m,) or C.shape != (n,):
         raise ValueError("shape mismatch")
-    rowsq = np.empty(m)
+    rowsq = np.empty(max(m, 1))
     colsq = np.empty(n)
     rc = lib().orc_step_matrix(m, n, _f64(X, "X"), _f64(P, "P"), _f64(R, "R"), _f64(C, "C"),
                                _f64(G, "G"), float(h), hp.alpha, hp.mu, hp.gamma, hp.eps_stab,

@@ -77,7 +77,8 @@ int orc_step_matrix(int64_t m, int64_t n, double *X, double *P, double *R, doubl
                     const double *G, double h, double alpha, double mu, double gamma,
                     double eps_stab, double *rowsq, double *colsq)
 {
-    if (m < 1 || n < 1 || !hparams_ok(h, alpha, mu, gamma, eps_stab))
+    /* m = 0 is an empty matrix: no momentum, and C only decays. */
+    if (m < 0 || n < 1 || !hparams_ok(h, alpha, mu, gamma, eps_stab))
         return ORC_EARG;
     const int64_t N = m * n;
 
@@ -151,7 +152,7 @@ int orc_step_matrix(int64_t m, int64_t n, double *X, double *P, double *R, doubl
 int orc_step_vector(int64_t L, double *x, double *p, double *xi, const double *g, double h,
                     double alpha, double mu, double gamma)
 {
-    if (L < 1 || !hparams_ok(h, alpha, mu, gamma, 0.0))
+    if (L < 0 || !hparams_ok(h, alpha, mu, gamma, 0.0))
         return ORC_EARG;
 
     /* B */

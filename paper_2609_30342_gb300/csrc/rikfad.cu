@@ -1,0 +1,766 @@
+// rikfad.cu -- C ABI of the R-iKFAD optimiser on GB300 (sm_103a): handle,
+// argument checking, device state, and the launches of the step kernels.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "rikfad.h"
+#include "rikfad_kernels.cuh"
+#include "rikfad_planner.hpp"
+
+using namespace rikfad;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const std::string &msg)
+{
+    g_last_error = msg;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what)
+{
+    g_last_error = std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+    return RIKFAD_ERR_CUDA;
+}
+
+#define RK_CUDA(call, what)                                   \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess)                                \
+            return cuda_fail(e_, what);                       \
+    } while (0)
+
+constexpr uint64_t kImageTag = 0x31444146694b5221ull;   // "!RKiFAD1"
+constexpr size_t kImageHeader = 64;
+
+struct ImageHeader {
+    uint64_t tag;
+    int64_t ntensors;
+    double pending_step;
+    int64_t fac_floats;
+    double alpha, mu, gamma, eps_stab;
+};
+static_assert(sizeof(ImageHeader) <= kImageHeader, "header too large");
+
+// A device table of per-tensor pointers, uploaded only when it changes.
+struct PtrTable {
+    int count = 0;                  // pointers in the table
+    void **dev = nullptr;
+    void **pinned = nullptr;        // staging for the host-to-device copy
+    std::vector<void *> cached;
+    bool valid = false;
+    cudaEvent_t uploaded = nullptr;
+};
+
+}  // namespace
+
+struct rikfad_handle_s {
+    int device = 0;
+    int ntensors = 0;
+    int grad_bytes = 4;
+    rikfad_hparams hp{};
+    Plan plan;
+    int max_blocks = 1;
+    double pending_step = 0.0;      // h_prev
+    std::vector<rikfad_shape> shapes;
+
+    // device memory
+    TensorDev *d_tensors = nullptr;
+    PanelDev *d_panels = nullptr;
+    PieceDev *d_pieces = nullptr;
+    int32_t *d_block_piece = nullptr;
+    int64_t *d_slot_off = nullptr;
+    FinItemDev *d_fin = nullptr;
+    float *d_fac = nullptr;
+    float *d_rowpart = nullptr;
+    float *d_colpart = nullptr;
+    float *d_spart = nullptr;
+    float *d_den = nullptr;
+    float *h_den = nullptr;         // pinned
+    size_t workspace = 0;
+
+    PtrTable step_ptrs;             // x | grad | p
+    PtrTable canon_ptrs;            // src | dst
+
+    bool profiling = false;
+    std::vector<cudaEvent_t> prof_events;   // 3 per recorded step
+    size_t prof_used = 0;
+};
+
+namespace {
+
+int check_handle(rikfad_handle h)
+{
+    if (h == nullptr)
+        return fail(RIKFAD_ERR_ARG, "handle is NULL");
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "cudaGetDevice");
+    if (dev != h->device)
+        return fail(RIKFAD_ERR_STATE, "current CUDA device " + std::to_string(dev) +
+                                          " differs from the handle's device " +
+                                          std::to_string(h->device));
+    return RIKFAD_OK;
+}
+
+template <typename T>
+int upload(T **dst, const std::vector<T> &src, size_t &bytes)
+{
+    *dst = nullptr;
+    if (src.empty())
+        return RIKFAD_OK;
+    const size_t nb = src.size() * sizeof(T);
+    cudaError_t e = cudaMalloc((void **)dst, nb);
+    if (e != cudaSuccess)
+        return e == cudaErrorMemoryAllocation ? fail(RIKFAD_ERR_OOM, "cudaMalloc of a plan table failed")
+                                              : cuda_fail(e, "cudaMalloc");
+    bytes += nb;
+    RK_CUDA(cudaMemcpy(*dst, src.data(), nb, cudaMemcpyHostToDevice), "cudaMemcpy plan table");
+    return RIKFAD_OK;
+}
+
+int alloc_zero(float **dst, int64_t floats, size_t &bytes)
+{
+    *dst = nullptr;
+    if (floats <= 0)
+        return RIKFAD_OK;
+    const size_t nb = (size_t)floats * sizeof(float);
+    cudaError_t e = cudaMalloc((void **)dst, nb);
+    if (e != cudaSuccess)
+        return e == cudaErrorMemoryAllocation ? fail(RIKFAD_ERR_OOM, "cudaMalloc failed")
+                                              : cuda_fail(e, "cudaMalloc");
+    bytes += nb;
+    RK_CUDA(cudaMemset(*dst, 0, nb), "cudaMemset");
+    return RIKFAD_OK;
+}
+
+int ptrtable_init(PtrTable &t, int count, size_t &bytes)
+{
+    t.count = count;
+    t.cached.assign(count, nullptr);
+    t.valid = false;
+    if (count == 0)
+        return RIKFAD_OK;
+    cudaError_t e = cudaMalloc((void **)&t.dev, sizeof(void *) * count);
+    if (e != cudaSuccess)
+        return fail(RIKFAD_ERR_OOM, "cudaMalloc of the pointer table failed");
+    bytes += sizeof(void *) * count;
+    e = cudaMallocHost((void **)&t.pinned, sizeof(void *) * count);
+    if (e != cudaSuccess)
+        return fail(RIKFAD_ERR_OOM, "cudaMallocHost of the pointer staging failed");
+    RK_CUDA(cudaEventCreateWithFlags(&t.uploaded, cudaEventDisableTiming), "cudaEventCreate");
+    return RIKFAD_OK;
+}
+
+void ptrtable_free(PtrTable &t)
+{
+    if (t.dev)
+        cudaFree(t.dev);
+    if (t.pinned)
+        cudaFreeHost(t.pinned);
+    if (t.uploaded)
+        cudaEventDestroy(t.uploaded);
+    t = PtrTable();
+}
+
+// Make the device table equal `want`; enqueue the copy on `stream` if needed.
+int ptrtable_set(PtrTable &t, const std::vector<void *> &want, cudaStream_t stream)
+{
+    if (t.count == 0 || (t.valid && want == t.cached))
+        return RIKFAD_OK;
+    // The staging buffer may still feed the previous copy.
+    RK_CUDA(cudaEventSynchronize(t.uploaded), "cudaEventSynchronize (pointer staging)");
+    std::memcpy(t.pinned, want.data(), sizeof(void *) * t.count);
+    RK_CUDA(cudaMemcpyAsync(t.dev, t.pinned, sizeof(void *) * t.count, cudaMemcpyHostToDevice, stream),
+            "cudaMemcpyAsync pointer table");
+    RK_CUDA(cudaEventRecord(t.uploaded, stream), "cudaEventRecord");
+    t.cached = want;
+    t.valid = true;
+    return RIKFAD_OK;
+}
+
+bool hparams_ok(const rikfad_hparams &hp, std::string &why)
+{
+    if (!(std::isfinite(hp.alpha) && hp.alpha > 0)) {
+        why = "alpha must be finite and > 0";
+        return false;
+    }
+    if (!(hp.mu > 0) || std::isnan(hp.mu)) {
+        why = "mu must be > 0";
+        return false;
+    }
+    if (!(std::isfinite(hp.gamma) && hp.gamma >= 0)) {
+        why = "gamma must be finite and >= 0";
+        return false;
+    }
+    if (!(std::isfinite(hp.eps_stab) && hp.eps_stab >= 0)) {
+        why = "eps_stab must be finite and >= 0";
+        return false;
+    }
+    return true;
+}
+
+void release(rikfad_handle h)
+{
+    cudaFree(h->d_tensors);
+    cudaFree(h->d_panels);
+    cudaFree(h->d_pieces);
+    cudaFree(h->d_block_piece);
+    cudaFree(h->d_slot_off);
+    cudaFree(h->d_fin);
+    cudaFree(h->d_fac);
+    cudaFree(h->d_rowpart);
+    cudaFree(h->d_colpart);
+    cudaFree(h->d_spart);
+    cudaFree(h->d_den);
+    if (h->h_den)
+        cudaFreeHost(h->h_den);
+    ptrtable_free(h->step_ptrs);
+    ptrtable_free(h->canon_ptrs);
+    for (cudaEvent_t ev : h->prof_events)
+        cudaEventDestroy(ev);
+    delete h;
+}
+
+// Alignment a tensor's pointers need: 16 bytes for the 8-wide paths,
+// natural alignment otherwise.
+bool aligned_for(const TensorDev &td, const void *ptr, size_t natural)
+{
+    const uintptr_t v = (uintptr_t)ptr;
+    const bool wide = td.cols == 0 || td.vec;
+    return (v % (wide ? 16 : natural)) == 0;
+}
+
+int64_t numel(const TensorDev &td) { return td.cols == 0 ? td.rows : td.rows * td.cols; }
+
+template <typename GT>
+void launch_step(const StepParams &p, bool reuse, int nblocks, cudaStream_t s)
+{
+    if (reuse)
+        rikfad_step_kernel<GT, true><<<nblocks, kThreads, 0, s>>>(p);
+    else
+        rikfad_step_kernel<GT, false><<<nblocks, kThreads, 0, s>>>(p);
+}
+
+int finalize(rikfad_handle h, float decay, float gain, int resum_only, cudaStream_t stream)
+{
+    if (h->plan.fin_items.empty())
+        return RIKFAD_OK;
+    FinParams f{};
+    f.tensors = h->d_tensors;
+    f.panels = h->d_panels;
+    f.items = h->d_fin;
+    f.slot_off = h->d_slot_off;
+    f.fac = h->d_fac;
+    f.rowpart = h->d_rowpart;
+    f.colpart = h->d_colpart;
+    f.spart = h->d_spart;
+    f.decay = decay;
+    f.gain = gain;
+    f.resum_only = resum_only;
+    rikfad_finalize_kernel<<<(unsigned)h->plan.fin_items.size(), kFinThreads, 0, stream>>>(f);
+    RK_CUDA(cudaGetLastError(), "launch rikfad_finalize_kernel");
+    return RIKFAD_OK;
+}
+
+int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool commit,
+              cudaStream_t stream)
+{
+    const int T = h->ntensors;
+    std::vector<void *> want(2 * (size_t)T);
+    for (int t = 0; t < T; ++t) {
+        const TensorDev &td = h->plan.tensors[t];
+        const bool empty = numel(td) == 0;
+        if (!empty && (src[t] == nullptr || dst[t] == nullptr))
+            return fail(RIKFAD_ERR_ARG, "momentum pointer of tensor " + std::to_string(t) + " is NULL");
+        if (!empty && (!aligned_for(td, src[t], 4) || !aligned_for(td, dst[t], 4)))
+            return fail(RIKFAD_ERR_ALIGN, "momentum pointer of tensor " + std::to_string(t) +
+                                              " is not aligned");
+        if (!commit && !empty && src[t] == dst[t] && td.cols != 0)
+            return fail(RIKFAD_ERR_ARG, "out must not alias p");
+        want[t] = (void *)src[t];
+        want[T + t] = (void *)dst[t];
+    }
+    if (h->plan.nblocks > 0) {
+        int rc = ptrtable_set(h->canon_ptrs, want, stream);
+        if (rc)
+            return rc;
+        CanonParams c{};
+        c.tensors = h->d_tensors;
+        c.panels = h->d_panels;
+        c.pieces = h->d_pieces;
+        c.block_piece = h->d_block_piece;
+        c.src = (const float *const *)h->canon_ptrs.dev;
+        c.dst = (float *const *)(h->canon_ptrs.dev + T);
+        c.fac = h->d_fac;
+        c.spart = h->d_spart;
+        c.ex_prev = (float)(-0.5 * h->pending_step * M_LOG2E);
+        c.damp_prev = (float)std::exp(-h->hp.gamma * h->pending_step);
+        c.eps = (float)h->hp.eps_stab;
+        rikfad_canonical_kernel<<<h->plan.nblocks, kThreads, 0, stream>>>(c);
+        RK_CUDA(cudaGetLastError(), "launch rikfad_canonical_kernel");
+    }
+    if (commit)
+        h->pending_step = 0.0;
+    return RIKFAD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+RIKFAD_API const char *rikfad_last_error(void) { return g_last_error.c_str(); }
+
+RIKFAD_API int rikfad_abi_version(void) { return 1; }
+
+RIKFAD_API size_t rikfad_state_bytes_for(const rikfad_shape *shapes, int ntensors, int include_momentum)
+{
+    if (!check_shapes(shapes, ntensors).empty())
+        return 0;
+    size_t scalars = 0;
+    for (int t = 0; t < ntensors; ++t) {
+        const int64_t m = shapes[t].rows, n = shapes[t].cols;
+        if (n == 0)
+            scalars += (size_t)m + (include_momentum ? (size_t)m : 0);
+        else
+            scalars += (size_t)(m + n) + (include_momentum ? (size_t)(m * n) : 0);
+    }
+    return scalars * sizeof(float);
+}
+
+RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, int grad_dtype,
+                                     int nctas, int64_t *out, int64_t cap)
+{
+    if (grad_dtype != RIKFAD_GRAD_F32 && grad_dtype != RIKFAD_GRAD_BF16)
+        return fail(RIKFAD_ERR_ARG, "grad_dtype must be RIKFAD_GRAD_F32 or RIKFAD_GRAD_BF16");
+    if (cap > 0 && out == nullptr)
+        return fail(RIKFAD_ERR_ARG, "out is NULL");
+    Plan plan;
+    std::string err = build_plan(shapes, ntensors, grad_dtype == RIKFAD_GRAD_BF16 ? 2 : 4, nctas, plan);
+    if (!err.empty())
+        return fail(RIKFAD_ERR_ARG, err);
+    int64_t row = 0;
+    for (int b = 0; b < plan.nblocks; ++b) {
+        for (int q = plan.block_piece[b]; q < plan.block_piece[b + 1]; ++q, ++row) {
+            if (row >= cap)
+                continue;
+            const PieceDev &pc = plan.pieces[q];
+            int64_t *r = out + row * 8;
+            r[0] = b;
+            r[1] = pc.tensor;
+            r[2] = pc.kind;
+            r[3] = pc.kind == kMatrixRows ? plan.panels[pc.panel].col0 : 0;
+            r[4] = pc.kind == kMatrixRows ? plan.panels[pc.panel].width : 0;
+            r[5] = pc.begin;
+            r[6] = pc.end;
+            r[7] = pc.slot;
+        }
+    }
+    return row;
+}
+
+RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
+                             int grad_dtype, rikfad_handle *out)
+{
+    if (out == nullptr)
+        return fail(RIKFAD_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (hp == nullptr)
+        return fail(RIKFAD_ERR_ARG, "hp is NULL");
+    std::string why;
+    if (!hparams_ok(*hp, why))
+        return fail(RIKFAD_ERR_ARG, why);
+    if (grad_dtype != RIKFAD_GRAD_F32 && grad_dtype != RIKFAD_GRAD_BF16)
+        return fail(RIKFAD_ERR_ARG, "grad_dtype must be RIKFAD_GRAD_F32 or RIKFAD_GRAD_BF16");
+    why = check_shapes(shapes, ntensors);
+    if (!why.empty())
+        return fail(RIKFAD_ERR_ARG, why);
+
+    int dev = 0, sms = 0, occ = 0;
+    RK_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+    RK_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+    // Persistent grid: as many blocks as can be resident at once.
+    int occ_min = 1 << 30;
+    const void *kernels[4] = {(const void *)rikfad_step_kernel<float, true>,
+                              (const void *)rikfad_step_kernel<float, false>,
+                              (const void *)rikfad_step_kernel<__nv_bfloat16, true>,
+                              (const void *)rikfad_step_kernel<__nv_bfloat16, false>};
+    for (const void *k : kernels) {
+        RK_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, 0),
+                "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+        occ_min = std::min(occ_min, occ);
+    }
+    if (occ_min < 1)
+        return fail(RIKFAD_ERR_CUDA, "step kernel cannot be resident on this device");
+
+    rikfad_handle h = new rikfad_handle_s();
+    h->device = dev;
+    h->ntensors = ntensors;
+    h->grad_bytes = grad_dtype == RIKFAD_GRAD_BF16 ? 2 : 4;
+    h->hp = *hp;
+    h->shapes.assign(shapes, shapes + ntensors);
+    h->max_blocks = sms * occ_min;
+    why = build_plan(shapes, ntensors, h->grad_bytes, h->max_blocks, h->plan);
+    if (!why.empty()) {
+        delete h;
+        return fail(RIKFAD_ERR_ARG, why);
+    }
+    const Plan &p = h->plan;
+    size_t ws = 0;
+    int rc = RIKFAD_OK;
+    if (!rc) rc = upload(&h->d_tensors, p.tensors, ws);
+    if (!rc) rc = upload(&h->d_panels, p.panels, ws);
+    if (!rc) rc = upload(&h->d_pieces, p.pieces, ws);
+    if (!rc) rc = upload(&h->d_block_piece, p.block_piece, ws);
+    if (!rc) rc = upload(&h->d_slot_off, p.slot_off, ws);
+    if (!rc) rc = upload(&h->d_fin, p.fin_items, ws);
+    size_t state = 0;
+    if (!rc) rc = alloc_zero(&h->d_fac, p.fac_floats, state);
+    if (!rc) rc = alloc_zero(&h->d_rowpart, p.rowpart_floats, ws);
+    if (!rc) rc = alloc_zero(&h->d_colpart, p.colpart_floats, ws);
+    if (!rc) rc = alloc_zero(&h->d_spart, p.spart_floats, ws);
+    if (!rc) rc = alloc_zero(&h->d_den, std::max(ntensors, 1), ws);
+    if (!rc && cudaMallocHost((void **)&h->h_den, sizeof(float) * std::max(ntensors, 1)) != cudaSuccess)
+        rc = fail(RIKFAD_ERR_OOM, "cudaMallocHost failed");
+    if (!rc) rc = ptrtable_init(h->step_ptrs, 3 * ntensors, ws);
+    if (!rc) rc = ptrtable_init(h->canon_ptrs, 2 * ntensors, ws);
+    if (!rc) {
+        cudaError_t e = cudaDeviceSynchronize();
+        if (e != cudaSuccess)
+            rc = cuda_fail(e, "cudaDeviceSynchronize after create");
+    }
+    if (rc) {
+        std::string msg = g_last_error;
+        release(h);
+        g_last_error = msg;
+        return rc;
+    }
+    h->workspace = ws;
+    *out = h;
+    return RIKFAD_OK;
+}
+
+RIKFAD_API void rikfad_destroy(rikfad_handle h)
+{
+    if (h == nullptr)
+        return;
+    const int dev = h->device;
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != dev)
+        cudaSetDevice(dev);
+    cudaDeviceSynchronize();
+    release(h);
+    if (cur >= 0 && cur != dev)
+        cudaSetDevice(cur);
+}
+
+RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const void *const *grad,
+                           float *const *p, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (!(std::isfinite(step) && step > 0))
+        return fail(RIKFAD_ERR_ARG, "step must be finite and > 0");
+    const int T = h->ntensors;
+    if (T > 0 && (x == nullptr || grad == nullptr || p == nullptr))
+        return fail(RIKFAD_ERR_ARG, "pointer array is NULL");
+    const double decay_d = std::exp(-h->hp.alpha * step);
+    const double gain_d = std::isinf(h->hp.mu) ? 0.0 : -std::expm1(-h->hp.alpha * step) / (h->hp.mu * h->hp.alpha);
+    if (!std::isfinite((float)gain_d))
+        return fail(RIKFAD_ERR_ARG, "(1 - e^{-alpha h})/(mu alpha) overflows float32");
+    std::vector<void *> want(3 * (size_t)T);
+    for (int t = 0; t < T; ++t) {
+        const TensorDev &td = h->plan.tensors[t];
+        if (numel(td) == 0) {
+            want[t] = want[T + t] = want[2 * T + t] = nullptr;
+            continue;
+        }
+        if (x[t] == nullptr || grad[t] == nullptr || p[t] == nullptr)
+            return fail(RIKFAD_ERR_ARG, "pointer of tensor " + std::to_string(t) + " is NULL");
+        if (!aligned_for(td, x[t], 4) || !aligned_for(td, p[t], 4) ||
+            !aligned_for(td, grad[t], (size_t)h->grad_bytes))
+            return fail(RIKFAD_ERR_ALIGN, "pointer of tensor " + std::to_string(t) +
+                                              " is not 16-byte aligned");
+        want[t] = x[t];
+        want[T + t] = (void *)grad[t];
+        want[2 * T + t] = p[t];
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    RK_CUDA(cudaPeekAtLastError(), "earlier CUDA error");
+    if (h->plan.nblocks > 0) {
+        rc = ptrtable_set(h->step_ptrs, want, s);
+        if (rc)
+            return rc;
+    }
+    cudaEvent_t *ev = nullptr;
+    if (h->profiling) {
+        if (h->prof_used + 3 > h->prof_events.size()) {
+            for (int i = 0; i < 3; ++i) {
+                cudaEvent_t e;
+                RK_CUDA(cudaEventCreate(&e), "cudaEventCreate");
+                h->prof_events.push_back(e);
+            }
+        }
+        ev = &h->prof_events[h->prof_used];
+        h->prof_used += 3;
+        RK_CUDA(cudaEventRecord(ev[0], s), "cudaEventRecord");
+    }
+    if (h->plan.nblocks > 0) {
+        StepParams a{};
+        a.tensors = h->d_tensors;
+        a.panels = h->d_panels;
+        a.pieces = h->d_pieces;
+        a.block_piece = h->d_block_piece;
+        a.xptr = (float *const *)h->step_ptrs.dev;
+        a.gptr = (const void *const *)(h->step_ptrs.dev + T);
+        a.pptr = (float *const *)(h->step_ptrs.dev + 2 * T);
+        a.fac = h->d_fac;
+        a.rowpart = h->d_rowpart;
+        a.colpart = h->d_colpart;
+        a.spart = h->d_spart;
+        a.h = (float)step;
+        a.ex_cur = (float)(-0.5 * step * M_LOG2E);
+        a.ex_prev = (float)(-0.5 * h->pending_step * M_LOG2E);
+        a.damp_prev = (float)std::exp(-h->hp.gamma * h->pending_step);
+        a.damp_cur = (float)std::exp(-h->hp.gamma * step);
+        a.decay = (float)decay_d;
+        a.gain = (float)gain_d;
+        a.eps = (float)h->hp.eps_stab;
+        const bool reuse = (step == h->pending_step);
+        if (h->grad_bytes == 2)
+            launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s);
+        else
+            launch_step<float>(a, reuse, h->plan.nblocks, s);
+        RK_CUDA(cudaGetLastError(), "launch rikfad_step_kernel");
+    }
+    if (ev)
+        RK_CUDA(cudaEventRecord(ev[1], s), "cudaEventRecord");
+    rc = finalize(h, (float)decay_d, (float)gain_d, 0, s);
+    if (rc)
+        return rc;
+    if (ev)
+        RK_CUDA(cudaEventRecord(ev[2], s), "cudaEventRecord");
+    h->pending_step = step;
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_materialize(rikfad_handle h, float *const *p, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (h->ntensors > 0 && p == nullptr)
+        return fail(RIKFAD_ERR_ARG, "p is NULL");
+    return canonical(h, (const float *const *)p, p, true, (cudaStream_t)stream);
+}
+
+RIKFAD_API int rikfad_canonical_momentum(rikfad_handle h, const float *const *p, float *const *out,
+                                         void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (h->ntensors > 0 && (p == nullptr || out == nullptr))
+        return fail(RIKFAD_ERR_ARG, "p or out is NULL");
+    return canonical(h, p, out, false, (cudaStream_t)stream);
+}
+
+RIKFAD_API size_t rikfad_state_bytes(rikfad_handle h, int include_momentum)
+{
+    if (h == nullptr)
+        return 0;
+    return rikfad_state_bytes_for(h->shapes.data(), h->ntensors, include_momentum);
+}
+
+RIKFAD_API size_t rikfad_workspace_bytes(rikfad_handle h) { return h ? h->workspace : 0; }
+
+RIKFAD_API double rikfad_pending_step(rikfad_handle h) { return h ? h->pending_step : 0.0; }
+
+RIKFAD_API int rikfad_get_factors(rikfad_handle h, int t, float *R_host, float *C_host)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (t < 0 || t >= h->ntensors)
+        return fail(RIKFAD_ERR_ARG, "tensor index out of range");
+    const TensorDev &td = h->plan.tensors[t];
+    RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    if (R_host && td.rows > 0)
+        RK_CUDA(cudaMemcpy(R_host, h->d_fac + td.fac_off, sizeof(float) * td.rows, cudaMemcpyDeviceToHost),
+                "cudaMemcpy factors");
+    if (C_host && td.cols > 0)
+        RK_CUDA(cudaMemcpy(C_host, h->d_fac + td.fac_off + td.rows, sizeof(float) * td.cols,
+                           cudaMemcpyDeviceToHost),
+                "cudaMemcpy factors");
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_set_factors(rikfad_handle h, int t, const float *R_host, const float *C_host)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (t < 0 || t >= h->ntensors)
+        return fail(RIKFAD_ERR_ARG, "tensor index out of range");
+    const TensorDev &td = h->plan.tensors[t];
+    const int64_t nr = td.rows, nc = td.cols;
+    for (int64_t i = 0; R_host && i < nr; ++i)
+        if (!(std::isfinite(R_host[i]) && R_host[i] >= 0))
+            return fail(RIKFAD_ERR_ARG, "factor values must be finite and >= 0");
+    for (int64_t j = 0; C_host && j < nc; ++j)
+        if (!(std::isfinite(C_host[j]) && C_host[j] >= 0))
+            return fail(RIKFAD_ERR_ARG, "factor values must be finite and >= 0");
+    RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    if (R_host && nr > 0)
+        RK_CUDA(cudaMemcpy(h->d_fac + td.fac_off, R_host, sizeof(float) * nr, cudaMemcpyHostToDevice),
+                "cudaMemcpy factors");
+    if (C_host && nc > 0)
+        RK_CUDA(cudaMemcpy(h->d_fac + td.fac_off + nr, C_host, sizeof(float) * nc, cudaMemcpyHostToDevice),
+                "cudaMemcpy factors");
+    rc = finalize(h, 1.f, 0.f, 1, 0);
+    if (rc)
+        return rc;
+    RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (host_out == nullptr)
+        return fail(RIKFAD_ERR_ARG, "host_out is NULL");
+    const int T = h->ntensors;
+    if (T == 0)
+        return RIKFAD_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    DenParams d{h->d_tensors, h->d_spart, h->d_den, T};
+    const int warps = 8;
+    rikfad_denominators_kernel<<<(T + warps - 1) / warps, 32 * warps, 0, s>>>(d);
+    RK_CUDA(cudaGetLastError(), "launch rikfad_denominators_kernel");
+    RK_CUDA(cudaMemcpyAsync(h->h_den, h->d_den, sizeof(float) * T, cudaMemcpyDeviceToHost, s),
+            "cudaMemcpyAsync denominators");
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    std::memcpy(host_out, h->h_den, sizeof(float) * T);
+    return RIKFAD_OK;
+}
+
+RIKFAD_API size_t rikfad_state_image_bytes(rikfad_handle h)
+{
+    return h ? kImageHeader + sizeof(float) * (size_t)h->plan.fac_floats : 0;
+}
+
+RIKFAD_API int rikfad_export_state(rikfad_handle h, void *dev_dst, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (dev_dst == nullptr)
+        return fail(RIKFAD_ERR_ARG, "dev_dst is NULL");
+    if ((uintptr_t)dev_dst % 16)
+        return fail(RIKFAD_ERR_ALIGN, "dev_dst must be 16-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    ImageHeader hd{};
+    hd.tag = kImageTag;
+    hd.ntensors = h->ntensors;
+    hd.pending_step = h->pending_step;
+    hd.fac_floats = h->plan.fac_floats;
+    hd.alpha = h->hp.alpha;
+    hd.mu = h->hp.mu;
+    hd.gamma = h->hp.gamma;
+    hd.eps_stab = h->hp.eps_stab;
+    // The header is small; a synchronous copy keeps the host struct's lifetime simple.
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    RK_CUDA(cudaMemcpy(dev_dst, &hd, sizeof hd, cudaMemcpyHostToDevice), "cudaMemcpy image header");
+    if (h->plan.fac_floats > 0)
+        RK_CUDA(cudaMemcpyAsync((char *)dev_dst + kImageHeader, h->d_fac, sizeof(float) * h->plan.fac_floats,
+                                cudaMemcpyDeviceToDevice, s),
+                "cudaMemcpyAsync image");
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_import_state(rikfad_handle h, const void *dev_src, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (dev_src == nullptr)
+        return fail(RIKFAD_ERR_ARG, "dev_src is NULL");
+    if ((uintptr_t)dev_src % 16)
+        return fail(RIKFAD_ERR_ALIGN, "dev_src must be 16-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    ImageHeader hd{};
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    RK_CUDA(cudaMemcpy(&hd, dev_src, sizeof hd, cudaMemcpyDeviceToHost), "cudaMemcpy image header");
+    if (hd.tag != kImageTag)
+        return fail(RIKFAD_ERR_ARG, "not an R-iKFAD state image");
+    if (hd.ntensors != h->ntensors || hd.fac_floats != h->plan.fac_floats)
+        return fail(RIKFAD_ERR_ARG, "state image was exported for other shapes");
+    if (hd.alpha != h->hp.alpha || hd.mu != h->hp.mu || hd.gamma != h->hp.gamma ||
+        hd.eps_stab != h->hp.eps_stab)
+        return fail(RIKFAD_ERR_ARG, "state image was exported with other hyperparameters");
+    if (h->plan.fac_floats > 0)
+        RK_CUDA(cudaMemcpyAsync(h->d_fac, (const char *)dev_src + kImageHeader,
+                                sizeof(float) * h->plan.fac_floats, cudaMemcpyDeviceToDevice, s),
+                "cudaMemcpyAsync image");
+    rc = finalize(h, 1.f, 0.f, 1, s);
+    if (rc)
+        return rc;
+    h->pending_step = hd.pending_step;
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_profile_enable(rikfad_handle h, int enable)
+{
+    if (h == nullptr)
+        return fail(RIKFAD_ERR_ARG, "handle is NULL");
+    h->profiling = enable != 0;
+    h->prof_used = 0;
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_profile_read(rikfad_handle h, double *step_kernel_ms, double *finalize_kernel_ms,
+                                   int64_t *steps)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    double a = 0, b = 0;
+    for (size_t i = 0; i + 3 <= h->prof_used; i += 3) {
+        float t1 = 0, t2 = 0;
+        RK_CUDA(cudaEventSynchronize(h->prof_events[i + 2]), "cudaEventSynchronize");
+        RK_CUDA(cudaEventElapsedTime(&t1, h->prof_events[i], h->prof_events[i + 1]), "cudaEventElapsedTime");
+        RK_CUDA(cudaEventElapsedTime(&t2, h->prof_events[i + 1], h->prof_events[i + 2]),
+                "cudaEventElapsedTime");
+        a += t1;
+        b += t2;
+    }
+    if (step_kernel_ms)
+        *step_kernel_ms = a;
+    if (finalize_kernel_ms)
+        *finalize_kernel_ms = b;
+    if (steps)
+        *steps = (int64_t)(h->prof_used / 3);
+    h->prof_used = 0;
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_launches_per_step(rikfad_handle h)
+{
+    if (h == nullptr)
+        return 0;
+    return (h->plan.nblocks > 0 ? 1 : 0) + (h->plan.fin_items.empty() ? 0 : 1);
+}
+
+}  // extern "C"

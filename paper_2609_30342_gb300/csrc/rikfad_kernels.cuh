@@ -1,0 +1,493 @@
+// rikfad_kernels.cuh -- sm_103a kernels of the R-iKFAD optimiser step.
+//
+// The method (BACD splitting, Appendix A of the paper):
+//   B  P^(B) = P_n - h G
+//   A  X_{n+1} = X_n + h P^(B)
+//   C  P^(1) = P^(B) exp(-(h/2) xi~_n),  xi~ = R C^T / (1^T R + eps)   (Eq. xi_def)
+//      R_{n+1} = e^{-alpha h} R_n + k [P^(1)]^2 1_n,  k = (1 - e^{-alpha h})/(mu alpha)
+//      C_{n+1} = e^{-alpha h} C_n + k ([P^(1)]^2)^T 1_m
+//      P^(2) = P^(1) exp(-(h/2) xi~_{n+1})
+//   D  P_{n+1} = P^(2) e^{-gamma h}
+//
+// Scheduling.  R_{n+1}, C_{n+1} are reductions over the whole matrix, so
+// P^(2) cannot be formed in the same pass that produces P^(1).  The step
+// kernel therefore stores P^(1) and the NEXT step applies the pending factor
+// exp(-(h_prev/2) xi~_{n+1}) e^{-gamma h_prev} on the fly, with the factors
+// that the finalise kernel of this step wrote.  Every element is read once
+// and written once per step (grad, X, P read; X, P written).  When the step
+// size does not change, the pending factor and this step's first half-damp
+// are the same exponential and one exp2 serves both.
+//
+// Reductions are deterministic: a warp owns a row segment (row sums by a
+// fixed shuffle tree), each lane owns fixed columns (column sums accumulate
+// row by row in lane-private shared memory, then across warps in warp order,
+// then across the blocks of a panel in slot order in the finalise kernel).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "rikfad_plan.hpp"
+
+namespace rikfad {
+
+struct StepParams {
+    const TensorDev *tensors;
+    const PanelDev *panels;
+    const PieceDev *pieces;
+    const int32_t *block_piece;
+    float *const *xptr;        // ntensors device pointers
+    const void *const *gptr;
+    float *const *pptr;
+    float *fac;                // R, C of matrices; friction of vectors
+    float *rowpart;
+    float *colpart;
+    const float *spart;        // partial sums of R (denominators)
+    float h;                   // step size
+    float ex_cur;              // -(h/2) log2(e): exp(-(h/2) xi) = exp2(ex_cur xi)
+    float ex_prev;             // -(h_prev/2) log2(e)
+    float damp_prev;           // e^{-gamma h_prev}
+    float damp_cur;            // e^{-gamma h} (vectors finish D inside the step)
+    float decay;               // e^{-alpha h}
+    float gain;                // (1 - e^{-alpha h})/(mu alpha)
+    float eps;                 // eps_stab
+};
+
+struct FinParams {
+    const TensorDev *tensors;
+    const PanelDev *panels;
+    const FinItemDev *items;
+    const int64_t *slot_off;
+    float *fac;
+    const float *rowpart;
+    const float *colpart;
+    float *spart;
+    float decay;
+    float gain;
+    int resum_only;            // 1: only recompute the partial sums of R
+};
+
+struct CanonParams {
+    const TensorDev *tensors;
+    const PanelDev *panels;
+    const PieceDev *pieces;
+    const int32_t *block_piece;
+    const float *const *src;
+    float *const *dst;
+    const float *fac;
+    const float *spart;
+    float ex_prev;
+    float damp_prev;
+    float eps;
+};
+
+struct DenParams {
+    const TensorDev *tensors;
+    const float *spart;
+    float *out;
+    int ntensors;
+};
+
+// ---------------------------------------------------------------- helpers
+
+__device__ __forceinline__ float warp_sum(float v)
+{
+    // Butterfly: float addition is commutative, so every lane ends with the
+    // bitwise-same total.
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// 1^T R of a matrix from the finalise kernel's partial sums, in a fixed order
+// (identical in every warp that computes it).
+__device__ __forceinline__ float row_total(const float *spart, const TensorDev &td)
+{
+    const int lane = threadIdx.x & 31;
+    float v = 0.f;
+    for (int c = lane; c < td.spart_cnt; c += 32)
+        v += spart[td.spart_off + c];
+    return warp_sum(v);
+}
+
+// 1 / (1^T R + eps), with the friction set to zero when the denominator is
+// zero (eps = 0 and R = 0; Theorem 3's convention).
+__device__ __forceinline__ float inv_denominator(float s, float eps)
+{
+    const float den = s + eps;
+    return den == 0.f ? 0.f : 1.f / den;
+}
+
+template <typename GT> struct Grad8;
+
+template <> struct Grad8<float> {
+    float v[8];
+    __device__ __forceinline__ void load(const float *g)
+    {
+        const float4 a = __ldcs(reinterpret_cast<const float4 *>(g));
+        const float4 b = __ldcs(reinterpret_cast<const float4 *>(g) + 1);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    __device__ __forceinline__ float get(int e) const { return v[e]; }
+};
+
+template <> struct Grad8<__nv_bfloat16> {
+    uint32_t w[4];
+    __device__ __forceinline__ void load(const __nv_bfloat16 *g)
+    {
+        const uint4 a = __ldcs(reinterpret_cast<const uint4 *>(g));
+        w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+    }
+    // bf16 -> f32 is exact: the bf16 bits are the high half of the f32.
+    __device__ __forceinline__ float get(int e) const
+    {
+        const uint32_t word = w[e >> 1];
+        return __uint_as_float((e & 1) ? (word & 0xffff0000u) : (word << 16));
+    }
+};
+
+__device__ __forceinline__ float grad_at(const float *g, int64_t i) { return __ldcs(g + i); }
+__device__ __forceinline__ float grad_at(const __nv_bfloat16 *g, int64_t i)
+{
+    return __bfloat162float(g[i]);
+}
+
+__device__ __forceinline__ void load8(const float *p, float (&v)[8])
+{
+    const float4 a = __ldcs(reinterpret_cast<const float4 *>(p));
+    const float4 b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+__device__ __forceinline__ void store8(float *p, const float (&v)[8])
+{
+    __stcs(reinterpret_cast<float4 *>(p), make_float4(v[0], v[1], v[2], v[3]));
+    __stcs(reinterpret_cast<float4 *>(p) + 1, make_float4(v[4], v[5], v[6], v[7]));
+}
+
+// ------------------------------------------- one element, matrix rule
+//
+// p_hat is the stored P^(1) of the previous step.  Returns P^(1) of this step
+// and updates x.  e_cur = exp(-(h/2) xi~_ij), e_prev = exp(-(h_prev/2) xi~_ij),
+// both with the current factors (= R_{n}, C_{n} of this step).
+__device__ __forceinline__ float matrix_element(float &x, float p_hat, float g, float e_cur,
+                                                float e_prev, const StepParams &a)
+{
+    const float p_n = (p_hat * e_prev) * a.damp_prev;   // pending C half-damp, then D
+    const float p_b = fmaf(-a.h, g, p_n);                 // B
+    x = fmaf(a.h, p_b, x);                                // A
+    return p_b * e_cur;                                   // C, first half-damp
+}
+
+// ------------------------------------------------- matrix piece, 8-wide
+
+template <typename GT, bool REUSE>
+__device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const PieceDev &pc,
+                                                 const TensorDev &td, const PanelDev &pd,
+                                                 const float *Cs, float *red, float inv)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t n = td.cols;
+    const int w = pd.width;
+    float *X = a.xptr[pc.tensor];
+    const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
+    float *P = a.pptr[pc.tensor];
+    const float *R = a.fac + td.fac_off;
+    float *rowpart = a.rowpart + td.rowpart_off + (int64_t)(pc.panel - td.panel0) * td.rows;
+    float *myred = red + warp * kPanelMax;
+
+    for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
+        const float rhat = R[row] * inv;
+        const float a_cur = a.ex_cur * rhat;
+        const float a_prev = REUSE ? a_cur : a.ex_prev * rhat;
+        const int64_t base = row * n + pd.col0;
+
+        // Two 256-column chunks at a time: every load of the pair is issued
+        // before any arithmetic on it.
+        float racc = 0.f;
+#pragma unroll 1
+        for (int g0 = 0; g0 < pd.nch; g0 += 2) {
+            float xv[2][8], pv[2][8];
+            Grad8<GT> gv[2];
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int c = (g0 + k) * kChunk + lane * 8;
+                if (c < w) {
+                    gv[k].load(G + base + c);
+                    load8(X + base + c, xv[k]);
+                    load8(P + base + c, pv[k]);
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int c = (g0 + k) * kChunk + lane * 8;
+                if (c < w) {
+                    const float4 c0 = *reinterpret_cast<const float4 *>(Cs + c);
+                    const float4 c1 = *reinterpret_cast<const float4 *>(Cs + c + 4);
+                    const float cv[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                    float q[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float e_cur = exp2f(a_cur * cv[e]);
+                        const float e_prev = REUSE ? e_cur : exp2f(a_prev * cv[e]);
+                        const float p1 = matrix_element(xv[k][e], pv[k][e], gv[k].get(e), e_cur,
+                                                        e_prev, a);
+                        pv[k][e] = p1;
+                        q[e] = p1 * p1;
+                        racc += q[e];
+                    }
+                    store8(X + base + c, xv[k]);
+                    store8(P + base + c, pv[k]);
+                    float4 *r4 = reinterpret_cast<float4 *>(myred + c);
+                    float4 r0 = r4[0], r1 = r4[1];
+                    r0.x += q[0]; r0.y += q[1]; r0.z += q[2]; r0.w += q[3];
+                    r1.x += q[4]; r1.y += q[5]; r1.z += q[6]; r1.w += q[7];
+                    r4[0] = r0;
+                    r4[1] = r1;
+                }
+            }
+        }
+        racc = warp_sum(racc);
+        if (lane == 0)
+            rowpart[row] = racc;
+    }
+}
+
+// ----------------------------------------------- matrix piece, scalar
+// For matrices whose rows are not 8-aligned (cols % 8 != 0).
+
+template <typename GT, bool REUSE>
+__device__ __forceinline__ void matrix_piece_scalar(const StepParams &a, const PieceDev &pc,
+                                                    const TensorDev &td, const PanelDev &pd,
+                                                    const float *Cs, float *red, float inv)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t n = td.cols;
+    const int w = pd.width;
+    float *X = a.xptr[pc.tensor];
+    const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
+    float *P = a.pptr[pc.tensor];
+    const float *R = a.fac + td.fac_off;
+    float *rowpart = a.rowpart + td.rowpart_off + (int64_t)(pc.panel - td.panel0) * td.rows;
+    float *myred = red + warp * kPanelMax;
+
+    for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
+        const float rhat = R[row] * inv;
+        const float a_cur = a.ex_cur * rhat;
+        const float a_prev = REUSE ? a_cur : a.ex_prev * rhat;
+        const int64_t base = row * n + pd.col0;
+        float racc = 0.f;
+        for (int c = lane; c < w; c += 32) {
+            const float e_cur = exp2f(a_cur * Cs[c]);
+            const float e_prev = REUSE ? e_cur : exp2f(a_prev * Cs[c]);
+            float x = X[base + c];
+            const float p1 = matrix_element(x, P[base + c], grad_at(G, base + c), e_cur, e_prev, a);
+            X[base + c] = x;
+            P[base + c] = p1;
+            const float q = p1 * p1;
+            racc += q;
+            myred[c] += q;
+        }
+        racc = warp_sum(racc);
+        if (lane == 0)
+            rowpart[row] = racc;
+    }
+}
+
+// ------------------------------------------ element-wise rule (vectors)
+//
+// Element-wise iKFAD (Section 2, "Memory Complexity"): the friction xi of the
+// element is local, so the whole step -- including the second half-damp and
+// D -- completes here and P holds P_{n+1}.
+__device__ __forceinline__ void vector_element(float &x, float &p, float &xi, float g,
+                                               const StepParams &a)
+{
+    const float p_b = fmaf(-a.h, g, p);                       // B
+    x = fmaf(a.h, p_b, x);                                    // A
+    const float p1 = p_b * exp2f(a.ex_cur * xi);              // C, first half-damp
+    xi = fmaf(a.gain, p1 * p1, a.decay * xi);                 // C, friction filter
+    p = (p1 * exp2f(a.ex_cur * xi)) * a.damp_cur;             // C, second half-damp; D
+}
+
+template <typename GT>
+__device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev &pc,
+                                             const TensorDev &td)
+{
+    float *X = a.xptr[pc.tensor];
+    const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
+    float *P = a.pptr[pc.tensor];
+    float *XI = a.fac + td.fac_off;
+    const int64_t b0 = pc.begin;                // multiple of 8 (planner)
+    const int64_t nvec = (pc.end - b0) / 8;
+    for (int64_t v = threadIdx.x; v < nvec; v += kThreads) {
+        const int64_t e0 = b0 + v * 8;
+        Grad8<GT> g;
+        g.load(G + e0);
+        float x[8], p[8], xi[8];
+        load8(X + e0, x);
+        load8(P + e0, p);
+        load8(XI + e0, xi);
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            vector_element(x[e], p[e], xi[e], g.get(e), a);
+        store8(X + e0, x);
+        store8(P + e0, p);
+        store8(XI + e0, xi);
+    }
+    for (int64_t e = b0 + nvec * 8 + threadIdx.x; e < pc.end; e += kThreads) {
+        float x = X[e], p = P[e], xi = XI[e];
+        vector_element(x, p, xi, grad_at(G, e), a);
+        X[e] = x;
+        P[e] = p;
+        XI[e] = xi;
+    }
+}
+
+// ------------------------------------------------------ the step kernel
+
+template <typename GT, bool REUSE>
+__global__ void __launch_bounds__(kThreads, 2) rikfad_step_kernel(StepParams a)
+{
+    __shared__ __align__(16) float Cs[kPanelMax];
+    __shared__ __align__(16) float red[kWarps * kPanelMax];
+    const int b = blockIdx.x;
+    const int q0 = a.block_piece[b], q1 = a.block_piece[b + 1];
+    for (int q = q0; q < q1; ++q) {
+        const PieceDev pc = a.pieces[q];
+        const TensorDev td = a.tensors[pc.tensor];
+        if (pc.kind == kElements) {
+            vector_piece<GT>(a, pc, td);
+            continue;
+        }
+        const PanelDev pd = a.panels[pc.panel];
+        const int w = pd.width;
+        // Stage this panel's C, clear the column accumulators.
+        const float *C = a.fac + td.fac_off + td.rows + pd.col0;
+        for (int c = threadIdx.x; c < w; c += kThreads)
+            Cs[c] = C[c];
+        for (int i = threadIdx.x; i < kWarps * kPanelMax; i += kThreads)
+            red[i] = 0.f;
+        const float inv = inv_denominator(row_total(a.spart, td), a.eps);
+        __syncthreads();
+        if (td.vec) {
+            matrix_piece_vec<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
+        } else {
+            matrix_piece_scalar<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
+        }
+        __syncthreads();
+        // Column partial sums of this piece, warps added in order.
+        float *out = a.colpart + pc.colpart_off;
+        for (int c = threadIdx.x; c < w; c += kThreads) {
+            float s = 0.f;
+#pragma unroll
+            for (int wi = 0; wi < kWarps; ++wi)
+                s += red[wi * kPanelMax + c];
+            out[c] = s;
+        }
+        __syncthreads();
+    }
+}
+
+// ---------------------------------------------------- finalise kernel
+//
+// R_{n+1} = e^{-alpha h} R_n + k sum_panels rowpart,
+// C_{n+1} = e^{-alpha h} C_n + k sum_slots colpart (slot order),
+// and the partial sums of R_{n+1} that give 1^T R_{n+1}.
+__global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams f)
+{
+    __shared__ float wsum[kFinThreads / 32];
+    const FinItemDev it = f.items[blockIdx.x];
+    const TensorDev td = f.tensors[it.tensor];
+    if (it.kind == kFinRows) {
+        const int64_t i = it.begin + threadIdx.x;
+        float val = 0.f;
+        if (i < it.end) {
+            float *R = f.fac + td.fac_off;
+            if (f.resum_only) {
+                val = R[i];
+            } else {
+                float acc = 0.f;
+                const float *rp = f.rowpart + td.rowpart_off + i;
+                for (int k = 0; k < td.npanels; ++k)
+                    acc += rp[(int64_t)k * td.rows];
+                val = fmaf(f.gain, acc, f.decay * R[i]);
+                R[i] = val;
+            }
+        }
+        val = warp_sum(val);
+        if ((threadIdx.x & 31) == 0)
+            wsum[threadIdx.x >> 5] = val;
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            float v = threadIdx.x < kFinThreads / 32 ? wsum[threadIdx.x] : 0.f;
+            v = warp_sum(v);
+            if (threadIdx.x == 0)
+                f.spart[td.spart_off + it.chunk] = v;
+        }
+    } else if (!f.resum_only) {
+        const PanelDev pd = f.panels[it.panel];
+        const int64_t c = it.begin + threadIdx.x;
+        if (c < it.end) {
+            float acc = 0.f;
+            for (int s = pd.slot_begin; s < pd.slot_end; ++s)
+                acc += f.colpart[f.slot_off[s] + c];
+            float *C = f.fac + td.fac_off + td.rows + pd.col0;
+            C[c] = fmaf(f.gain, acc, f.decay * C[c]);
+        }
+    }
+}
+
+// ------------------------------------------- canonical momentum kernel
+//
+// dst = src exp(-(h_prev/2) xi~) e^{-gamma h_prev} for matrices (the same
+// expression, in the same rounding order, as the start of the next step);
+// vectors already hold P_{n+1} and are copied when dst != src.
+__global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams c)
+{
+    __shared__ float Cs[kPanelMax];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int q0 = c.block_piece[blockIdx.x], q1 = c.block_piece[blockIdx.x + 1];
+    for (int q = q0; q < q1; ++q) {
+        const PieceDev pc = c.pieces[q];
+        const TensorDev td = c.tensors[pc.tensor];
+        const float *S = c.src[pc.tensor];
+        float *D = c.dst[pc.tensor];
+        if (pc.kind == kElements) {
+            if (S != D)
+                for (int64_t e = pc.begin + threadIdx.x; e < pc.end; e += kThreads)
+                    D[e] = S[e];
+            continue;
+        }
+        const PanelDev pd = c.panels[pc.panel];
+        const float *C = c.fac + td.fac_off + td.rows + pd.col0;
+        for (int j = threadIdx.x; j < pd.width; j += kThreads)
+            Cs[j] = C[j];
+        const float inv = inv_denominator(row_total(c.spart, td), c.eps);
+        __syncthreads();
+        const float *R = c.fac + td.fac_off;
+        for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
+            const float a_prev = c.ex_prev * (R[row] * inv);
+            const int64_t base = row * td.cols + pd.col0;
+            for (int j = lane; j < pd.width; j += 32)
+                D[base + j] = (S[base + j] * exp2f(a_prev * Cs[j])) * c.damp_prev;
+        }
+        __syncthreads();
+    }
+}
+
+// 1^T R of every matrix (0 for vectors), same summation order as the kernels.
+__global__ void rikfad_denominators_kernel(DenParams d)
+{
+    const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    if (t >= d.ntensors)
+        return;
+    const TensorDev td = d.tensors[t];
+    const float s = td.cols == 0 ? 0.f : row_total(d.spart, td);
+    if ((threadIdx.x & 31) == 0)
+        d.out[t] = s;
+}
+
+}  // namespace rikfad

@@ -1,0 +1,213 @@
+// rikfad_planner.cpp -- host-side work plan of the fused R-iKFAD step.
+#include "rikfad_planner.hpp"
+
+#include <algorithm>
+#include <cstdint>
+#include <cstdio>
+#include <limits>
+
+namespace rikfad {
+
+namespace {
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
+
+struct Unit {
+    int32_t kind;
+    int32_t tensor;
+    int32_t panel;
+    int64_t len;    // rows or elements
+    int64_t cost;   // bytes per row or element
+    int64_t gran;   // cut granularity
+};
+
+}  // namespace
+
+std::string check_shapes(const rikfad_shape *shapes, int ntensors)
+{
+    if (ntensors < 0)
+        return "ntensors is negative";
+    if (ntensors > 0 && shapes == nullptr)
+        return "shapes is NULL";
+    const int64_t kMaxCols = std::numeric_limits<int32_t>::max() / 2;
+    for (int t = 0; t < ntensors; ++t) {
+        const int64_t m = shapes[t].rows, n = shapes[t].cols;
+        char buf[160];
+        if (m < 0 || n < 0) {
+            snprintf(buf, sizeof buf, "tensor %d: negative shape (%lld, %lld)", t, (long long)m,
+                     (long long)n);
+            return buf;
+        }
+        if (n > kMaxCols) {
+            snprintf(buf, sizeof buf, "tensor %d: cols %lld exceeds %lld", t, (long long)n,
+                     (long long)kMaxCols);
+            return buf;
+        }
+        if (n > 0 && m > (std::numeric_limits<int64_t>::max() / 64) / n) {
+            snprintf(buf, sizeof buf, "tensor %d: rows x cols overflows", t);
+            return buf;
+        }
+    }
+    return "";
+}
+
+std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes, int max_blocks,
+                       Plan &plan)
+{
+    std::string err = check_shapes(shapes, ntensors);
+    if (!err.empty())
+        return err;
+    if (grad_bytes != 2 && grad_bytes != 4)
+        return "gradient element size must be 2 or 4 bytes";
+    if (max_blocks < 1)
+        return "block budget must be >= 1";
+    Plan p;
+    std::vector<Unit> units;
+
+    // Per-tensor layout: factor storage, column panels, row partials.
+    int64_t fac = 0, rowpart = 0;
+    int64_t spart = 0;
+    for (int t = 0; t < ntensors; ++t) {
+        TensorDev td{};
+        td.rows = shapes[t].rows;
+        td.cols = shapes[t].cols;
+        td.fac_off = fac;
+        td.panel0 = -1;
+        if (td.cols == 0) {
+            td.vec = 1;
+            fac += round_up(td.rows, 8);
+            if (td.rows > 0)
+                units.push_back({kElements, t, -1, td.rows, vector_elem_bytes(grad_bytes),
+                                 kElemGranule});
+        } else {
+            td.vec = (td.cols % 8 == 0) ? 1 : 0;
+            fac += round_up(td.rows + td.cols, 8);
+            int64_t np = ceil_div(td.cols, kPanelMax);
+            int64_t w = ceil_div(td.cols, np);
+            if (td.vec)
+                w = round_up(w, 8);
+            np = ceil_div(td.cols, w);
+            td.npanels = (int32_t)np;
+            td.panel0 = (int32_t)p.panels.size();
+            for (int64_t k = 0; k < np; ++k) {
+                PanelDev pd{};
+                pd.tensor = t;
+                pd.col0 = (int32_t)(k * w);
+                pd.width = (int32_t)std::min<int64_t>(w, td.cols - k * w);
+                pd.nch = (int32_t)ceil_div(pd.width, kChunk);
+                pd.slot_begin = pd.slot_end = 0;
+                if (td.rows > 0)
+                    units.push_back({kMatrixRows, t, (int32_t)p.panels.size(), td.rows,
+                                     pd.width * matrix_elem_bytes(grad_bytes), 1});
+                p.panels.push_back(pd);
+            }
+            td.rowpart_off = rowpart;
+            rowpart += td.rows * np;
+            td.spart_off = (int32_t)spart;
+            td.spart_cnt = (int32_t)ceil_div(td.rows, kFinThreads);
+            spart += td.spart_cnt;
+        }
+        p.tensors.push_back(td);
+    }
+    if (spart > std::numeric_limits<int32_t>::max())
+        return "too many rows";
+    p.fac_floats = fac;
+    p.rowpart_floats = rowpart;
+    p.spart_floats = (int32_t)spart;
+
+    int64_t total = 0;
+    for (const Unit &u : units)
+        total += u.len * u.cost;
+    p.total_bytes = total;
+
+    // Cut the unit sequence into nblocks shares of nearly equal cost.
+    p.block_piece.push_back(0);
+    if (total > 0) {
+        const int64_t G = std::min<int64_t>(max_blocks, std::max<int64_t>(1, ceil_div(total, kMinBlockBytes)));
+        p.nblocks = (int)G;
+        int64_t block = 0, acc = 0;
+        auto boundary = [&](int64_t b) { return (int64_t)((__int128)total * (b + 1) / G); };
+        int64_t bound = boundary(0);
+        int64_t colpart = 0;
+        for (const Unit &u : units) {
+            int64_t pos = 0;
+            while (pos < u.len) {
+                int64_t take;
+                if (block == G - 1) {
+                    take = u.len - pos;
+                } else {
+                    const int64_t room = bound - acc;
+                    take = room > 0 ? ceil_div(room, u.cost) : 1;
+                    take = round_up(take, u.gran);
+                    take = std::min(take, u.len - pos);
+                }
+                PieceDev pc{};
+                pc.kind = u.kind;
+                pc.tensor = u.tensor;
+                pc.panel = u.panel;
+                pc.begin = pos;
+                pc.end = pos + take;
+                pc.slot = -1;
+                pc.colpart_off = 0;
+                if (u.kind == kMatrixRows) {
+                    PanelDev &pd = p.panels[u.panel];
+                    const int32_t slot = (int32_t)p.slot_off.size();
+                    if (pd.slot_end == pd.slot_begin)
+                        pd.slot_begin = slot;
+                    pd.slot_end = slot + 1;
+                    pc.slot = slot;
+                    pc.colpart_off = colpart;
+                    p.slot_off.push_back(colpart);
+                    colpart += pd.width;
+                }
+                p.pieces.push_back(pc);
+                acc += take * u.cost;
+                pos += take;
+                while (acc >= bound && block < G - 1) {
+                    ++block;
+                    p.block_piece.push_back((int32_t)p.pieces.size());
+                    bound = boundary(block);
+                }
+            }
+        }
+        while ((int64_t)p.block_piece.size() < G + 1)
+            p.block_piece.push_back((int32_t)p.pieces.size());
+        p.colpart_floats = colpart;
+    }
+
+    // Finalise work: R in chunks of kFinThreads rows (each also yields one
+    // partial sum of R), C in chunks of kFinThreads columns of each panel.
+    for (int t = 0; t < ntensors; ++t) {
+        const TensorDev &td = p.tensors[t];
+        if (td.cols == 0)
+            continue;
+        for (int32_t c = 0; c < td.spart_cnt; ++c) {
+            FinItemDev it{};
+            it.kind = kFinRows;
+            it.tensor = t;
+            it.panel = -1;
+            it.chunk = c;
+            it.begin = (int64_t)c * kFinThreads;
+            it.end = std::min<int64_t>(td.rows, it.begin + kFinThreads);
+            p.fin_items.push_back(it);
+        }
+        for (int32_t k = 0; k < td.npanels; ++k) {
+            const PanelDev &pd = p.panels[td.panel0 + k];
+            for (int64_t c0 = 0; c0 < pd.width; c0 += kFinThreads) {
+                FinItemDev it{};
+                it.kind = kFinCols;
+                it.tensor = t;
+                it.panel = td.panel0 + k;
+                it.chunk = 0;
+                it.begin = c0;
+                it.end = std::min<int64_t>(pd.width, c0 + kFinThreads);
+                p.fin_items.push_back(it);
+            }
+        }
+    }
+    plan = std::move(p);
+    return "";
+}
+
+}  // namespace rikfad

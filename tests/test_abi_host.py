@@ -1,0 +1,132 @@
+"""The C-ABI library on the host: it loads, exports what the header declares,
+and its planner covers every element exactly once (CPU only, no GPU calls)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2609_30342_gb300 import build as pkg_build
+from paper_2609_30342_gb300 import rikfad, workloads
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "rikfad.h")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    pkg_build.build()
+    yield
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"RIKFAD_API\s+[\w\s\*]+?\b(rikfad_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for want in ("rikfad_create", "rikfad_step", "rikfad_state_bytes", "rikfad_destroy",
+                 "rikfad_materialize", "rikfad_last_error"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol():
+    L = ctypes.CDLL(rikfad.LIB_PATH)
+    for name in declared_symbols():
+        assert hasattr(L, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", rikfad.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\b(rikfad_\w+)\b", out))
+    assert exported == set(declared_symbols()), exported ^ set(declared_symbols())
+
+
+def test_binding_covers_every_declared_symbol():
+    bound = {name for name, _, _ in rikfad.SIGNATURES}
+    assert bound == set(declared_symbols())
+
+
+def test_abi_version_and_error_string():
+    assert rikfad.lib().rikfad_abi_version() == 1
+    assert isinstance(rikfad.lib().rikfad_last_error(), bytes)
+
+
+GPT2S = [s for _, s in workloads.gpt2_small()]
+NANO = [s for _, s in workloads.gpt2_nano()]
+ODD = [(1, 1), (1, 7), (3, 5), (257, 129), (0, 4), (5, 0), (0, 0), (13, 0), (9, 2048),
+       (2, 3000), (4096, 8), (100, 1032)]
+
+
+def _cost(shape, gb):
+    m, n = shape
+    return m * (gb + 24) if n == 0 else m * n * (gb + 16)
+
+
+@pytest.mark.parametrize("shapes", [GPT2S, NANO, ODD, workloads.SWEEP_SHAPES[:2], [(256, 512)]],
+                         ids=["gpt2s", "nano", "odd", "sweep", "single"])
+@pytest.mark.parametrize("nblocks", [1, 7, 304, 1216])
+@pytest.mark.parametrize("grad", ["bf16", "f32"])
+def test_plan_covers_every_element_once(shapes, nblocks, grad):
+    plan = rikfad.plan_query(shapes, grad, nblocks)
+    gb = 2 if grad == "bf16" else 4
+    blocks = plan[:, 0]
+    assert np.all(np.diff(blocks) >= 0), "pieces out of block order"
+    assert blocks.size == 0 or (blocks.min() >= 0 and blocks.max() < nblocks)
+    # Coverage: mark every (row, column) of every matrix and every element of
+    # every vector; each must be hit exactly once.
+    hits = [np.zeros(workloads.array_shape(s), np.int32) for s in shapes]
+    slots = []
+    for b, t, kind, col0, width, beg, end, slot in plan:
+        m, n = shapes[t]
+        assert beg < end
+        if kind == 0:
+            assert n > 0 and 0 <= beg and end <= m and 0 <= col0 and col0 + width <= n
+            assert width <= 1024
+            if n % 8 == 0:
+                assert col0 % 8 == 0 and width % 8 == 0
+            hits[t][beg:end, col0:col0 + width] += 1
+            slots.append(slot)
+        else:
+            assert n == 0 and 0 <= beg and end <= m and beg % 8 == 0
+            hits[t][beg:end] += 1
+    for t, hit in enumerate(hits):
+        assert np.all(hit == 1), "tensor %d covered %s times" % (t, np.unique(hit))
+    assert slots == list(range(len(slots))), "slots must be consecutive in piece order"
+    # Balance: no block exceeds its fair share by more than one unit of work.
+    if plan.size:
+        total = sum(_cost(s, gb) for s in shapes)
+        used = int(blocks.max()) + 1
+        per_block = np.zeros(used)
+        largest_unit = 0
+        for b, t, kind, col0, width, beg, end, slot in plan:
+            unit = width * (gb + 16) if kind == 0 else 8 * (gb + 24)
+            largest_unit = max(largest_unit, unit)
+            per_block[b] += (end - beg) * unit / (1 if kind == 0 else 8)
+        assert abs(per_block.sum() - total) < 1e-6 * total
+        fair = total / used
+        assert per_block.max() <= fair + 2 * largest_unit + 1, (per_block.max(), fair)
+
+
+def test_plan_rejects_bad_arguments():
+    with pytest.raises(rikfad.RikfadError):
+        rikfad.plan_query([(-1, 3)], "bf16", 10)
+    with pytest.raises(rikfad.RikfadError):
+        rikfad.plan_query([(3, 3)], "bf16", 0)
+
+
+def test_state_bytes_match_oracle_count():
+    for shapes in (GPT2S, NANO, ODD):
+        assert rikfad.state_bytes_for(shapes, True) == 4 * oracle.state_scalars(shapes)
+        N = workloads.count(shapes)[0]
+        assert rikfad.state_bytes_for(shapes, False) == 4 * (oracle.state_scalars(shapes) - N)
+
+
+def test_state_bytes_gpt2s_vs_full_friction():
+    """R-iKFAD on GPT2-S (split q/k/v): 4 (N + sum(m + n) + 1-D) bytes; full
+    iKFAD / Adam keep 2N floats."""
+    N, mats, mn, one_d = workloads.count(GPT2S)
+    assert (N, mats, mn, one_d) == (124439808, 74, 218705, 121344)
+    assert rikfad.state_bytes_for(GPT2S, True) == 4 * (N + mn + one_d) == 499119428

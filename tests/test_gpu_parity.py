@@ -1,0 +1,273 @@
+"""Parity of the CUDA path (through the C ABI) with the oracle, on seeded
+synthetic inputs.  Needs a GPU."""
+import multiprocessing as mp
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import HParams
+from paper_2609_30342_gb300 import build as pkg_build
+from paper_2609_30342_gb300 import rikfad, workloads
+
+import oracle_jobs
+from gpu_helpers import GpuRun, compare, compare_state, oracle_from_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    pkg_build.build()
+    oracle.lib()
+    yield
+
+
+# ---------------------------------------------------------------- config 1
+
+def _config1_hp():
+    return HParams(alpha=0.01, mu=1.0, gamma=0.0, eps_stab=1e-8)
+
+
+def test_single_matrix_every_step():
+    """256 x 512 fp32, fresh N(0, 0.01^2) gradient per step (seed 0), 10 steps:
+    the full state after every step against the oracle run alongside, plus
+    the one-step error from the GPU's own state (oracle re-seeded each step)."""
+    hp = _config1_hp()
+    h = 1e-3
+    X0, P0, G = workloads.single_matrix_inputs(256, 512, seed=0, steps=10)
+    shapes = [(256, 512)]
+    run = GpuRun(shapes, hp, False, [X0], [P0])
+    ref = oracle.ModelState(shapes, [X0], [P0])
+    for k in range(1, 11):
+        seeded = oracle_from_gpu(run)
+        run.set_grads([G[k - 1]])
+        run.step(h)
+        ref.step([G[k - 1].astype(np.float64)], h, hp)
+        seeded.step([G[k - 1].astype(np.float64)], h, hp)
+        if k == 1:
+            compare_state(run, ref, 1e-5, 1e-2, "step1 ")
+        else:
+            compare_state(run, ref, 1e-4, 1e-2, "step%d " % k)
+        compare_state(run, seeded, 1e-5, 1e-2, "reseeded step%d " % k)
+    run.close()
+
+
+def test_single_matrix_100_steps():
+    """Same matrix, 100 steps with a larger step size so the friction acts:
+    state within 1e-4 after 100 steps."""
+    hp = HParams(alpha=0.5, mu=1e-6, gamma=0.0, eps_stab=1e-8)
+    h = 0.05
+    X0, P0, G = workloads.single_matrix_inputs(256, 512, seed=0, steps=100)
+    shapes = [(256, 512)]
+    run = GpuRun(shapes, hp, False, [X0], [P0])
+    ref = oracle.ModelState(shapes, [X0], [P0])
+    for k in range(100):
+        run.set_grads([G[k]])
+        run.step(h)
+        ref.step([G[k].astype(np.float64)], h, hp)
+    compare_state(run, ref, 1e-4, 1e-2, "step100 ")
+    # the friction must have been doing something
+    R, C = run.factors()[0]
+    s = R.sum()
+    xi = np.outer(R, C) / (s + hp.eps_stab)
+    assert 0.5 * h * xi.max() > 1e-3
+    run.close()
+
+
+# ---------------------------------------------------------------- config 2
+
+QUAD = dict(m=1024, n=1024, seed=1, steps=2000, h=1e-3, alpha=0.01, mu=1.0, eps=1e-8)
+SNAPS = (1, 100, 2000)
+
+
+@pytest.fixture(scope="module")
+def quadratic_oracle():
+    ctx = mp.get_context("spawn")
+    pool = ctx.Pool(2)
+    jobs = {g: pool.apply_async(oracle_jobs.quadratic_run,
+                                (QUAD["m"], QUAD["n"], QUAD["seed"], QUAD["steps"], QUAD["h"],
+                                 QUAD["alpha"], QUAD["mu"], g, QUAD["eps"], SNAPS))
+            for g in (0.0, 0.1)}
+    yield jobs
+    pool.terminate()
+    pool.join()
+
+
+@pytest.mark.parametrize("gamma", [0.0, 0.1])
+def test_strongly_convex_quadratic(gamma, quadratic_oracle):
+    """f = 1/2 sum A (.) (X - X*)^2, A ~ U[0.1, 10], X* ~ N(0, 1) (seed 1),
+    1024 x 1024, 2000 steps: the paper's energy E = f - f* + 1/2 ||P||^2
+    (Section 3) decreases, X moves toward X*, and both trajectories agree
+    with the oracle."""
+    prob = workloads.QuadraticProblem(QUAD["m"], QUAD["n"], QUAD["seed"])
+    hp = HParams(QUAD["alpha"], QUAD["mu"], gamma, QUAD["eps"])
+    run = GpuRun([(QUAD["m"], QUAD["n"])], hp, False, [prob.X0], [prob.P0])
+    A = torch.from_numpy(prob.A).cuda()
+    Xs = torch.from_numpy(prob.Xstar).cuda()
+    A64, Xs64 = A.double(), Xs.double()
+    energy = []
+
+    def gpu_energy():
+        run.opt.canonical_momentum(run.p, run.out)
+        D = run.x[0].double() - Xs64
+        return float(0.5 * (A64 * D * D).sum() + 0.5 * (run.out[0].double() ** 2).sum())
+
+    energy.append(gpu_energy())
+    snaps, seeded = {}, None
+    for k in range(1, QUAD["steps"] + 1):
+        torch.mul(A, run.x[0] - Xs, out=run.g[0])      # gradient of the test objective
+        if k == QUAD["steps"]:
+            seeded = oracle_from_gpu(run)
+            seeded.step([run.g[0].double().cpu().numpy()], QUAD["h"], hp)
+        run.step(QUAD["h"])
+        energy.append(gpu_energy())
+        if k in SNAPS:
+            snaps[k] = (run.X()[0], run.canonical_P()[0]) + run.factors()[0]
+    ref_energy, ref_snaps = quadratic_oracle[gamma].get(timeout=1800)
+    energy = np.array(energy)
+    # energy: non-increasing along the GPU trajectory, and equal to the oracle's
+    assert np.all(np.diff(energy) <= 1e-7 * energy[:-1]), "energy increased"
+    assert energy[-1] < 0.5 * energy[0]
+    compare("energy", energy, ref_energy, 1e-4, 0.0)
+    dist0 = np.linalg.norm(prob.X0 - prob.Xstar)
+    assert np.linalg.norm(snaps[2000][0] - prob.Xstar) < dist0
+    # The last step alone, from the GPU's own state: 1e-5.
+    compare_state(run, seeded, 1e-5, 1e-2, "gamma%g reseeded step2000 " % gamma)
+    # Whole trajectories.  After 2000 steps the float32 rounding of X and P
+    # accumulated along the trajectory dominates: judge the state against the
+    # scale of each tensor (floor = its rms) at 1e-4.
+    failures = []
+    for k, rtol, floor in ((1, 1e-5, 1e-2), (100, 1e-4, 1e-2), (2000, 1e-4, 1.0)):
+        for name, g, r in zip("XPRC", snaps[k], ref_snaps[k]):
+            try:
+                compare("gamma%g step%d %s" % (gamma, k, name), g, r, rtol, floor)
+            except AssertionError as e:
+                failures.append(str(e))
+    assert not failures, "\n".join(failures)
+    run.close()
+
+
+# ------------------------------------------------------ ragged / edge cases
+
+EDGE_SHAPES = [(1, 1), (1, 7), (3, 5), (257, 129), (9, 2048), (2, 3000), (100, 1032), (4096, 8),
+               (5, 0), (13, 0), (0, 0), (0, 4), (3, 0), (37, 24), (1, 1024), (1025, 1),
+               (8, 1040), (64, 0)]
+
+
+@pytest.mark.parametrize("grad_bf16", [False, True])
+@pytest.mark.parametrize("eps,gamma", [(1e-8, 0.0), (0.25, 0.3), (0.0, 0.0)])
+def test_edge_shapes(grad_bf16, eps, gamma):
+    """Tiny, ragged and empty tensors in one list; factors start nonzero with
+    1^T R != 1^T C (so the placement of eps_stab on 1^T R matters), the step
+    size changes between steps (two exponentials per element) and returns.
+    With eps_stab = 0 the factors start at zero (Theorem 3's convention)."""
+    rng = np.random.default_rng(5)
+    shapes = EDGE_SHAPES
+    hp = HParams(alpha=0.3, mu=0.05, gamma=gamma, eps_stab=eps)
+    X = [rng.standard_normal(workloads.array_shape(s)).astype(np.float32) for s in shapes]
+    P = [(0.1 * rng.standard_normal(workloads.array_shape(s))).astype(np.float32) for s in shapes]
+    run = GpuRun(shapes, hp, grad_bf16, X, P)
+    if eps > 0:
+        for t, (m, n) in enumerate(shapes):
+            R = rng.uniform(0.0, 2.0, m).astype(np.float32)
+            C = rng.uniform(0.0, 0.5, n).astype(np.float32) if n else None
+            run.opt.set_factors(t, R, C)
+    ref = oracle_from_gpu(run)
+    for k, h in enumerate((0.05, 0.05, 0.11, 0.02, 0.02)):
+        g = [rng.standard_normal(workloads.array_shape(s)).astype(np.float32) for s in shapes]
+        if grad_bf16:
+            g = [workloads.bf16_round(a) for a in g]
+        seeded = oracle_from_gpu(run)
+        run.set_grads(g)
+        run.step(h)
+        g64 = [a.astype(np.float64) for a in g]
+        ref.step(g64, h, hp)
+        seeded.step(g64, h, hp)
+        compare_state(run, seeded, 1e-5, 1e-2, "reseeded step%d " % (k + 1))
+        compare_state(run, ref, 1e-4, 1e-2, "step%d " % (k + 1))
+    run.close()
+
+
+# ------------------------------------------------------------ model-sized
+
+def _model_parity(shapes, seed, hp, h, steps, tensors=None):
+    inp = workloads.ModelInputs(shapes, seed=seed)
+    run = GpuRun(shapes, hp, True, inp.X, inp.P)
+    ref = oracle.ModelState([shapes[t] for t in tensors] if tensors else shapes,
+                            [inp.X[t] for t in tensors] if tensors else inp.X,
+                            [inp.P[t] for t in tensors] if tensors else inp.P)
+    for k in range(steps):
+        g = inp.grads(k)
+        run.set_grads(g)
+        run.step(h)
+        sel = [g[t] for t in tensors] if tensors else g
+        ref.step([a.astype(np.float64) for a in sel], h, hp)
+    return run, ref
+
+
+def _subset_compare(run, ref, tensors, rtol, floor, tag):
+    Xg, Pg, F = run.X(), run.canonical_P(), run.factors()
+    for i, t in enumerate(tensors):
+        compare("%sX[%d]" % (tag, t), Xg[t], ref.X[i], rtol, floor)
+        compare("%sP[%d]" % (tag, t), Pg[t], ref.P[i], rtol, floor)
+        if run.shapes[t][1] == 0:
+            compare("%sxi[%d]" % (tag, t), F[t][0], ref.xi[i], rtol, floor)
+        else:
+            compare("%sR[%d]" % (tag, t), F[t][0], ref.R[i], rtol, floor)
+            compare("%sC[%d]" % (tag, t), F[t][1], ref.C[i], rtol, floor)
+
+
+GPT2S_HP = HParams(alpha=0.0579, mu=1.3637e-6, gamma=0.0, eps_stab=1e-16)
+GPT2S_H = 0.0918
+
+
+def test_gpt2_nano_shaped_full_model():
+    """GPT2-Nano-shaped list (6 x 384, vocab 50304; 100 tensors, 30.06M
+    parameters), bf16 gradients (seed 2), paper's GPT2-S hyperparameters:
+    every tensor against the oracle after 1 and after 3 steps."""
+    shapes = [s for _, s in workloads.gpt2_nano()]
+    run, ref = _model_parity(shapes, 2, GPT2S_HP, GPT2S_H, 1)
+    compare_state(run, ref, 1e-5, 1e-2, "nano step1 ")
+    inp = workloads.ModelInputs(shapes, seed=2)
+    for k in (1, 2):
+        g = inp.grads(k)
+        run.set_grads(g)
+        run.step(GPT2S_H)
+        ref.step([a.astype(np.float64) for a in g], GPT2S_H, GPT2S_HP)
+    compare_state(run, ref, 1e-4, 1e-2, "nano step3 ")
+    run.close()
+
+
+def test_gpt2_small_full_size():
+    """GPT2-S list (196 tensors, 124.4M parameters), bf16 gradients (seed 3),
+    in the launch configuration the benchmark times: the token embedding,
+    the first block and the final LayerNorm exactly against the oracle after
+    2 steps; every tensor checked for the proved invariants (R, C >= 0,
+    sum R = sum C from zero, finite state)."""
+    named = workloads.gpt2_small()
+    shapes = [s for _, s in named]
+    names = [n for n, _ in named]
+    pick = [i for i, n in enumerate(names) if n == "wte" or n.startswith("h0.") or
+            n.startswith("ln_f")]
+    run, ref = _model_parity(shapes, 3, GPT2S_HP, GPT2S_H, 2, tensors=pick)
+    _subset_compare(run, ref, pick, 1e-4, 1e-2, "gpt2s step2 ")
+    F = run.factors()
+    for t, (m, n) in enumerate(shapes):
+        if n == 0 or m == 0:
+            continue
+        R, C = F[t]
+        assert np.all(R >= 0) and np.all(C >= 0) and np.all(np.isfinite(R))
+        assert abs(R.sum() - C.sum()) <= 1e-4 * max(R.sum(), 1e-30), names[t]
+    for x in run.x:
+        assert torch.isfinite(x).all()
+    run.close()
+
+
+@pytest.mark.parametrize("shape", workloads.SWEEP_SHAPES, ids=lambda s: "%dx%d" % s)
+def test_large_matrix_sweep(shape):
+    """Tall, wide and square matrices (seed 4), 2 steps, full comparison."""
+    run, ref = _model_parity([shape], 4, GPT2S_HP, GPT2S_H, 2)
+    compare_state(run, ref, 1e-4, 1e-2, "%dx%d step2 " % shape)
+    run.close()
