@@ -219,6 +219,46 @@ RIKFAD_API int rikfad_launches_per_step(rikfad_handle h);
 RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, int grad_dtype,
                                      int nctas, int64_t *out, int64_t cap);
 
+/*
+ * Allocation-free step for one matrix.  This entry point has no counterpart
+ * in the paper; it is a convenience of this library.
+ *
+ * rikfad_create allocates the factors and a reduction workspace with
+ * cudaMalloc.  Some callers cannot allocate device memory on their own: a
+ * framework whose caching allocator already holds the GPU's memory (a second
+ * allocator next to it fails or fragments the pool), or a latency-bound
+ * service that allows no cudaMalloc after start-up because the call can
+ * synchronise the device and stall all its streams.  This call allocates
+ * nothing: the caller owns every input and output, and the partial sums live
+ * in a fixed 4.45 MB array compiled into the library, which every GPU that
+ * loads the library keeps until the process exits.
+ *
+ * It performs one rikfad_step on a single matrix in the same stored form:
+ *   rows, cols    0 <= rows <= 65536, 1 <= cols <= 1024 (anything larger is
+ *                 rejected with RIKFAD_ERR_ARG)
+ *   step          step size h > 0
+ *   pending_step  the step size of this matrix's previous call (0 for the
+ *                 first call, or after the momentum was made canonical);
+ *                 the caller keeps this number, the library keeps no state
+ *   hp            hyperparameters, as for rikfad_create
+ *   grad_dtype    RIKFAD_GRAD_F32 or RIKFAD_GRAD_BF16
+ *   x, grad, p    device, rows x cols row-major, as for rikfad_step (16-byte
+ *                 aligned when cols is a multiple of 8)
+ *   R, C          device, rows and cols floats: the factors, read and updated
+ *                 (start them at zero)
+ * The first call on each device looks up the array's device address (and
+ * may load the library's device code onto that GPU); make that first call
+ * before any stream capture.  Every call clears the array's counter before
+ * its launch and rewrites the partial sums, so calls in sequence are
+ * independent.  All calls share the one array: calls whose work overlaps on
+ * the GPU (unordered streams) race and give wrong results.  Errors as for
+ * rikfad_step, reported through rikfad_last_error.
+ */
+RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols, double step,
+                                          double pending_step, const rikfad_hparams *hp,
+                                          int grad_dtype, float *x, const void *grad, float *p,
+                                          float *R, float *C, void *stream);
+
 /* Last error message of the calling thread ("" if none). */
 RIKFAD_API const char *rikfad_last_error(void);
 

@@ -61,6 +61,15 @@ struct PtrTable {
 
 }  // namespace
 
+namespace rikfad {
+// Lets the library's other translation units report through rikfad_last_error.
+int report_error(int code, const std::string &msg)
+{
+    g_last_error = msg;
+    return code;
+}
+}  // namespace rikfad
+
 struct rikfad_handle_s {
     int device = 0;
     int ntensors = 0;

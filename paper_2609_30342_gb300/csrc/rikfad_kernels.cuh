@@ -391,6 +391,11 @@ __global__ void __launch_bounds__(kThreads, 2) rikfad_step_kernel(StepParams a)
     }
 }
 
+// The kernels below are defined once, in rikfad.cu; other translation units
+// that only reuse the device functions above define
+// RIKFAD_DEVICE_FUNCTIONS_ONLY before including this header.
+#ifndef RIKFAD_DEVICE_FUNCTIONS_ONLY
+
 // ---------------------------------------------------- finalise kernel
 //
 // R_{n+1} = e^{-alpha h} R_n + k sum_panels rowpart,
@@ -489,5 +494,7 @@ __global__ void rikfad_denominators_kernel(DenParams d)
     if ((threadIdx.x & 31) == 0)
         d.out[t] = s;
 }
+
+#endif  // RIKFAD_DEVICE_FUNCTIONS_ONLY
 
 }  // namespace rikfad

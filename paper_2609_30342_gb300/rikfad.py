@@ -69,6 +69,9 @@ SIGNATURES = [
     ("rikfad_plan_query", ctypes.c_int64, [ctypes.POINTER(Shape), ctypes.c_int, ctypes.c_int,
                                            ctypes.c_int, ctypes.POINTER(ctypes.c_int64),
                                            ctypes.c_int64]),
+    ("rikfad_step_matrix_noalloc", ctypes.c_int, [ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
+                                                  ctypes.c_double, ctypes.POINTER(HParams),
+                                                  ctypes.c_int, _VP, _VP, _VP, _VP, _VP, _VP]),
     ("rikfad_last_error", ctypes.c_char_p, []),
     ("rikfad_abi_version", ctypes.c_int, []),
 ]
@@ -144,6 +147,18 @@ def plan_query(shapes, grad_dtype, nblocks):
     if n2 != n:
         raise RuntimeError("plan size changed between calls")
     return out[:n]
+
+
+def step_matrix_noalloc(rows, cols, h, pending_step, alpha, mu, gamma, eps_stab, grad_dtype, x, grad,
+                        p, R, C, stream=None):
+    """One allocation-free step of a single matrix (``rikfad_step_matrix_noalloc``):
+    the caller owns x, grad, p and the factors R, C, and remembers the
+    previous step size itself (``pending_step``)."""
+    hp = HParams(float(alpha), float(mu), float(gamma), float(eps_stab))
+    gd = GRAD_BF16 if grad_dtype in ("bf16", GRAD_BF16) else GRAD_F32
+    _check(lib().rikfad_step_matrix_noalloc(int(rows), int(cols), float(h), float(pending_step),
+                                            ctypes.byref(hp), gd, _ptr(x), _ptr(grad), _ptr(p),
+                                            _ptr(R), _ptr(C), _stream_ptr(stream)))
 
 
 class PointerSet:
