@@ -9,7 +9,7 @@
 #include <vector>
 
 #include "rikfad.h"
-#include "rikfad_kernels.cuh"
+#include "rikfad_aux_kernels.cuh"
 #include "rikfad_planner.hpp"
 
 using namespace rikfad;

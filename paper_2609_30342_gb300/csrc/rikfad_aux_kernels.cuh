@@ -1,0 +1,160 @@
+// rikfad_aux_kernels.cuh -- the kernels around the step kernel: the factor
+// finalise (run after every step), the canonical-momentum pass (checkpoints,
+// tests) and the denominator read-back.  Included by rikfad.cu only.
+#pragma once
+#include "rikfad_kernels.cuh"
+
+namespace rikfad {
+
+struct DenParams {
+    const TensorDev *tensors;
+    const float *spart;
+    float *out;
+    int ntensors;
+};
+
+struct CanonParams {
+    const TensorDev *tensors;
+    const PanelDev *panels;
+    const PieceDev *pieces;
+    const int32_t *block_piece;
+    const float *const *src;
+    float *const *dst;
+    const float *fac;
+    const float *spart;
+    float ex_prev;
+    float damp_prev;
+    float eps;
+};
+
+struct FinParams {
+    const TensorDev *tensors;
+    const PanelDev *panels;
+    const FinItemDev *items;
+    const int64_t *slot_off;
+    float *fac;
+    const float *rowpart;
+    const float *colpart;
+    float *spart;
+    float decay;
+    float gain;
+    int resum_only;            // 1: only recompute the partial sums of R
+};
+
+
+// ---------------------------------------------------- finalise kernel
+//
+// R_{n+1} = e^{-alpha h} R_n + k sum_panels rowpart,
+// C_{n+1} = e^{-alpha h} C_n + k sum_slots colpart,
+// and the partial sums of R_{n+1} that give 1^T R_{n+1}.
+//
+// A row item is kFinThreads rows, one thread per row.  A column item is
+// kFinColChunk (32) columns of one panel: warp w adds the slots
+// slot_begin + w, + 8, ... for the 32 columns (coalesced 128-byte rows of the
+// partials), then warp 0 adds the eight warp sums in order.
+__global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams f)
+{
+    __shared__ float wsum[kFinThreads / 32];
+    __shared__ float csum[kFinThreads / 32][32];
+    const FinItemDev it = f.items[blockIdx.x];
+    const TensorDev td = f.tensors[it.tensor];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (it.kind == kFinRows) {
+        const int64_t i = it.begin + threadIdx.x;
+        float val = 0.f;
+        if (i < it.end) {
+            float *R = f.fac + td.fac_off;
+            if (f.resum_only) {
+                val = R[i];
+            } else {
+                float acc = 0.f;
+                const float *rp = f.rowpart + td.rowpart_off + i;
+                for (int k = 0; k < td.npanels; ++k)
+                    acc += rp[(int64_t)k * td.rows];
+                val = fmaf(f.gain, acc, f.decay * R[i]);
+                R[i] = val;
+            }
+        }
+        val = warp_sum(val);
+        if (lane == 0)
+            wsum[warp] = val;
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            float v = threadIdx.x < kFinThreads / 32 ? wsum[threadIdx.x] : 0.f;
+            v = warp_sum(v);
+            if (threadIdx.x == 0)
+                f.spart[td.spart_off + it.chunk] = v;
+        }
+    } else if (!f.resum_only) {
+        const PanelDev pd = f.panels[it.panel];
+        const int64_t c = it.begin + lane;
+        float acc = 0.f;
+        if (c < it.end) {
+#pragma unroll 4
+            for (int s = pd.slot_begin + warp; s < pd.slot_end; s += kFinThreads / 32)
+                acc += f.colpart[f.slot_off[s] + c];
+        }
+        csum[warp][lane] = acc;
+        __syncthreads();
+        if (warp == 0 && c < it.end) {
+            float t = 0.f;
+#pragma unroll
+            for (int k = 0; k < kFinThreads / 32; ++k)
+                t += csum[k][lane];
+            float *C = f.fac + td.fac_off + td.rows + pd.col0;
+            C[c] = fmaf(f.gain, t, f.decay * C[c]);
+        }
+    }
+}
+
+// ------------------------------------------- canonical momentum kernel
+//
+// dst = src exp(-(h_prev/2) xi~) e^{-gamma h_prev} for matrices (the same
+// expression, in the same rounding order, as the start of the next step);
+// vectors already hold P_{n+1} and are copied when dst != src.
+__global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams c)
+{
+    __shared__ float Cs[kPanelMax];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int q0 = c.block_piece[blockIdx.x], q1 = c.block_piece[blockIdx.x + 1];
+    for (int q = q0; q < q1; ++q) {
+        const PieceDev pc = c.pieces[q];
+        const TensorDev td = c.tensors[pc.tensor];
+        const float *S = c.src[pc.tensor];
+        float *D = c.dst[pc.tensor];
+        if (pc.kind == kElements) {
+            if (S != D)
+                for (int64_t e = pc.begin + threadIdx.x; e < pc.end; e += kThreads)
+                    D[e] = S[e];
+            continue;
+        }
+        const PanelDev pd = c.panels[pc.panel];
+        const float *C = c.fac + td.fac_off + td.rows + pd.col0;
+        for (int j = threadIdx.x; j < pd.width; j += kThreads)
+            Cs[j] = C[j];
+        const float inv = inv_denominator(row_total(c.spart, td), c.eps);
+        __syncthreads();
+        const float *R = c.fac + td.fac_off;
+        for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
+            const float a_prev = c.ex_prev * (R[row] * inv);
+            const int64_t base = row * td.cols + pd.col0;
+            for (int j = lane; j < pd.width; j += 32)
+                D[base + j] = (S[base + j] * exp2f(a_prev * Cs[j])) * c.damp_prev;
+        }
+        __syncthreads();
+    }
+}
+
+// 1^T R of every matrix (0 for vectors), same summation order as the kernels.
+__global__ void rikfad_denominators_kernel(DenParams d)
+{
+    const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    if (t >= d.ntensors)
+        return;
+    const TensorDev td = d.tensors[t];
+    const float s = td.cols == 0 ? 0.f : row_total(d.spart, td);
+    if ((threadIdx.x & 31) == 0)
+        d.out[t] = s;
+}
+
+}  // namespace rikfad

@@ -53,41 +53,6 @@ struct StepParams {
     float eps;                 // eps_stab
 };
 
-struct FinParams {
-    const TensorDev *tensors;
-    const PanelDev *panels;
-    const FinItemDev *items;
-    const int64_t *slot_off;
-    float *fac;
-    const float *rowpart;
-    const float *colpart;
-    float *spart;
-    float decay;
-    float gain;
-    int resum_only;            // 1: only recompute the partial sums of R
-};
-
-struct CanonParams {
-    const TensorDev *tensors;
-    const PanelDev *panels;
-    const PieceDev *pieces;
-    const int32_t *block_piece;
-    const float *const *src;
-    float *const *dst;
-    const float *fac;
-    const float *spart;
-    float ex_prev;
-    float damp_prev;
-    float eps;
-};
-
-struct DenParams {
-    const TensorDev *tensors;
-    const float *spart;
-    float *out;
-    int ntensors;
-};
-
 // ---------------------------------------------------------------- helpers
 
 __device__ __forceinline__ float warp_sum(float v)
@@ -184,6 +149,11 @@ __device__ __forceinline__ float matrix_element(float &x, float p_hat, float g, 
 
 // ------------------------------------------------- matrix piece, 8-wide
 
+// 256-column chunks whose loads are issued together (registers: ~20 per chunk).
+#ifndef RIKFAD_CHUNK_GROUP
+#define RIKFAD_CHUNK_GROUP 1
+#endif
+
 template <typename GT, bool REUSE>
 __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const PieceDev &pc,
                                                  const TensorDev &td, const PanelDev &pd,
@@ -205,15 +175,15 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
         const float a_prev = REUSE ? a_cur : a.ex_prev * rhat;
         const int64_t base = row * n + pd.col0;
 
-        // Two 256-column chunks at a time: every load of the pair is issued
-        // before any arithmetic on it.
+        // RIKFAD_CHUNK_GROUP 256-column chunks at a time: every load of the
+        // group is issued before any arithmetic on it.
         float racc = 0.f;
 #pragma unroll 1
-        for (int g0 = 0; g0 < pd.nch; g0 += 2) {
-            float xv[2][8], pv[2][8];
-            Grad8<GT> gv[2];
+        for (int g0 = 0; g0 < pd.nch; g0 += RIKFAD_CHUNK_GROUP) {
+            float xv[RIKFAD_CHUNK_GROUP][8], pv[RIKFAD_CHUNK_GROUP][8];
+            Grad8<GT> gv[RIKFAD_CHUNK_GROUP];
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
+            for (int k = 0; k < RIKFAD_CHUNK_GROUP; ++k) {
                 const int c = (g0 + k) * kChunk + lane * 8;
                 if (c < w) {
                     gv[k].load(G + base + c);
@@ -222,7 +192,7 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
                 }
             }
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
+            for (int k = 0; k < RIKFAD_CHUNK_GROUP; ++k) {
                 const int c = (g0 + k) * kChunk + lane * 8;
                 if (c < w) {
                     const float4 c0 = *reinterpret_cast<const float4 *>(Cs + c);
@@ -348,8 +318,13 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
 
 // ------------------------------------------------------ the step kernel
 
+// Blocks per SM the register budget is sized for (2: 128 registers/thread).
+#ifndef RIKFAD_STEP_MIN_BLOCKS
+#define RIKFAD_STEP_MIN_BLOCKS 2
+#endif
+
 template <typename GT, bool REUSE>
-__global__ void __launch_bounds__(kThreads, 2) rikfad_step_kernel(StepParams a)
+__global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_kernel(StepParams a)
 {
     __shared__ __align__(16) float Cs[kPanelMax];
     __shared__ __align__(16) float red[kWarps * kPanelMax];
@@ -390,111 +365,5 @@ __global__ void __launch_bounds__(kThreads, 2) rikfad_step_kernel(StepParams a)
         __syncthreads();
     }
 }
-
-// The kernels below are defined once, in rikfad.cu; other translation units
-// that only reuse the device functions above define
-// RIKFAD_DEVICE_FUNCTIONS_ONLY before including this header.
-#ifndef RIKFAD_DEVICE_FUNCTIONS_ONLY
-
-// ---------------------------------------------------- finalise kernel
-//
-// R_{n+1} = e^{-alpha h} R_n + k sum_panels rowpart,
-// C_{n+1} = e^{-alpha h} C_n + k sum_slots colpart (slot order),
-// and the partial sums of R_{n+1} that give 1^T R_{n+1}.
-__global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams f)
-{
-    __shared__ float wsum[kFinThreads / 32];
-    const FinItemDev it = f.items[blockIdx.x];
-    const TensorDev td = f.tensors[it.tensor];
-    if (it.kind == kFinRows) {
-        const int64_t i = it.begin + threadIdx.x;
-        float val = 0.f;
-        if (i < it.end) {
-            float *R = f.fac + td.fac_off;
-            if (f.resum_only) {
-                val = R[i];
-            } else {
-                float acc = 0.f;
-                const float *rp = f.rowpart + td.rowpart_off + i;
-                for (int k = 0; k < td.npanels; ++k)
-                    acc += rp[(int64_t)k * td.rows];
-                val = fmaf(f.gain, acc, f.decay * R[i]);
-                R[i] = val;
-            }
-        }
-        val = warp_sum(val);
-        if ((threadIdx.x & 31) == 0)
-            wsum[threadIdx.x >> 5] = val;
-        __syncthreads();
-        if (threadIdx.x < 32) {
-            float v = threadIdx.x < kFinThreads / 32 ? wsum[threadIdx.x] : 0.f;
-            v = warp_sum(v);
-            if (threadIdx.x == 0)
-                f.spart[td.spart_off + it.chunk] = v;
-        }
-    } else if (!f.resum_only) {
-        const PanelDev pd = f.panels[it.panel];
-        const int64_t c = it.begin + threadIdx.x;
-        if (c < it.end) {
-            float acc = 0.f;
-            for (int s = pd.slot_begin; s < pd.slot_end; ++s)
-                acc += f.colpart[f.slot_off[s] + c];
-            float *C = f.fac + td.fac_off + td.rows + pd.col0;
-            C[c] = fmaf(f.gain, acc, f.decay * C[c]);
-        }
-    }
-}
-
-// ------------------------------------------- canonical momentum kernel
-//
-// dst = src exp(-(h_prev/2) xi~) e^{-gamma h_prev} for matrices (the same
-// expression, in the same rounding order, as the start of the next step);
-// vectors already hold P_{n+1} and are copied when dst != src.
-__global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams c)
-{
-    __shared__ float Cs[kPanelMax];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int q0 = c.block_piece[blockIdx.x], q1 = c.block_piece[blockIdx.x + 1];
-    for (int q = q0; q < q1; ++q) {
-        const PieceDev pc = c.pieces[q];
-        const TensorDev td = c.tensors[pc.tensor];
-        const float *S = c.src[pc.tensor];
-        float *D = c.dst[pc.tensor];
-        if (pc.kind == kElements) {
-            if (S != D)
-                for (int64_t e = pc.begin + threadIdx.x; e < pc.end; e += kThreads)
-                    D[e] = S[e];
-            continue;
-        }
-        const PanelDev pd = c.panels[pc.panel];
-        const float *C = c.fac + td.fac_off + td.rows + pd.col0;
-        for (int j = threadIdx.x; j < pd.width; j += kThreads)
-            Cs[j] = C[j];
-        const float inv = inv_denominator(row_total(c.spart, td), c.eps);
-        __syncthreads();
-        const float *R = c.fac + td.fac_off;
-        for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
-            const float a_prev = c.ex_prev * (R[row] * inv);
-            const int64_t base = row * td.cols + pd.col0;
-            for (int j = lane; j < pd.width; j += 32)
-                D[base + j] = (S[base + j] * exp2f(a_prev * Cs[j])) * c.damp_prev;
-        }
-        __syncthreads();
-    }
-}
-
-// 1^T R of every matrix (0 for vectors), same summation order as the kernels.
-__global__ void rikfad_denominators_kernel(DenParams d)
-{
-    const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
-    if (t >= d.ntensors)
-        return;
-    const TensorDev td = d.tensors[t];
-    const float s = td.cols == 0 ? 0.f : row_total(d.spart, td);
-    if ((threadIdx.x & 31) == 0)
-        d.out[t] = s;
-}
-
-#endif  // RIKFAD_DEVICE_FUNCTIONS_ONLY
 
 }  // namespace rikfad

@@ -24,7 +24,6 @@
 #include <string>
 
 #include "rikfad.h"
-#define RIKFAD_DEVICE_FUNCTIONS_ONLY
 #include "rikfad_kernels.cuh"
 
 using namespace rikfad;

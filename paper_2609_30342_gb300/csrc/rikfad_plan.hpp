@@ -22,6 +22,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kPanelMax = 1024;      // widest column panel (floats staged in shared memory)
 constexpr int kChunk = 256;          // columns one warp covers per pass (32 lanes x 8)
 constexpr int kFinThreads = 256;     // threads of the finalise kernel (= rows per partial sum)
+constexpr int kFinColChunk = 32;     // columns per finalise column item
 constexpr int kElemGranule = 8;      // element pieces start on multiples of 8 elements
 constexpr int64_t kMinBlockBytes = 64 * 1024;   // smallest share worth a block
 

@@ -177,7 +177,7 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
     }
 
     // Finalise work: R in chunks of kFinThreads rows (each also yields one
-    // partial sum of R), C in chunks of kFinThreads columns of each panel.
+    // partial sum of R), C in chunks of kFinColChunk columns of each panel.
     for (int t = 0; t < ntensors; ++t) {
         const TensorDev &td = p.tensors[t];
         if (td.cols == 0)
@@ -194,14 +194,14 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
         }
         for (int32_t k = 0; k < td.npanels; ++k) {
             const PanelDev &pd = p.panels[td.panel0 + k];
-            for (int64_t c0 = 0; c0 < pd.width; c0 += kFinThreads) {
+            for (int64_t c0 = 0; c0 < pd.width; c0 += kFinColChunk) {
                 FinItemDev it{};
                 it.kind = kFinCols;
                 it.tensor = t;
                 it.panel = td.panel0 + k;
                 it.chunk = 0;
                 it.begin = c0;
-                it.end = std::min<int64_t>(pd.width, c0 + kFinThreads);
+                it.end = std::min<int64_t>(pd.width, c0 + kFinColChunk);
                 p.fin_items.push_back(it);
             }
         }
