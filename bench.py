@@ -66,12 +66,15 @@ def workload(name):
     return named, desc, seed
 
 
-def algorithmic_bytes(shapes, grad_bytes):
+def algorithmic_bytes(shapes, grad_bytes, method="rikfad"):
     """Compulsory HBM bytes of one step: every matrix element reads the
     gradient, X and P and writes X and P (grad + 16 bytes); every vector
-    element also reads and writes its friction (grad + 24 bytes)."""
+    element also reads and writes its friction (grad + 24 bytes).  Under
+    full-friction iKFAD every element is a vector element."""
     from paper_2609_30342_gb300 import workloads as W
     N, _, _, one_d = W.count(shapes)
+    if method == "ikfad":
+        return N * (grad_bytes + 24)
     return (N - one_d) * (grad_bytes + 16) + one_d * (grad_bytes + 24)
 
 
@@ -302,13 +305,17 @@ def run_ours(args, rank, world, local_rank):
     p = [torch.zeros(W.array_shape(s), dtype=torch.float32, device=dev) for s in shapes]
     del inp, grads
 
-    opt = rikfad.RIKFAD(shapes, grad_dtype="bf16", **HP)
+    hp = dict(HP, gamma=args.gamma)
+    opt = rikfad.RIKFAD(shapes, grad_dtype="bf16", method=args.method, **hp)
     ptrs = opt.pack(x, g_views, p)
     stream = torch.cuda.current_stream(dev)
-    alg_bytes = algorithmic_bytes(shapes, 2)
+    alg_bytes = algorithmic_bytes(shapes, 2, args.method)
+    # --vary-h alternates the step size, so every step applies a pending
+    # factor of a different h (two exponentials per matrix element).
+    hs = (STEP, 0.9 * STEP) if args.vary_h else (STEP, STEP)
 
-    for _ in range(args.warmup):
-        opt.step(STEP, ptrs=ptrs, stream=stream)
+    for i in range(args.warmup):
+        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
     torch.cuda.synchronize(dev)
 
     # ---- device-timed region: inputs resident in HBM (2.24 GB > 129 MB L2)
@@ -325,8 +332,8 @@ def run_ours(args, rank, world, local_rank):
     sampler.start()
     time.sleep(0.25)      # let the sampler take its first reading
     ev0.record(stream)
-    for _ in range(args.steps):
-        opt.step(STEP, ptrs=ptrs, stream=stream)
+    for i in range(args.steps):
+        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     clocks = sampler.stop()
@@ -347,9 +354,9 @@ def run_ours(args, rank, world, local_rank):
     barrier(world)
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
-    for _ in range(args.steps):
+    for i in range(args.steps):
         g_dev.copy_(g_host, non_blocking=True)
-        opt.step(STEP, ptrs=ptrs, stream=stream)
+        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
         opt.read_denominators(stream)
     torch.cuda.synchronize(dev)
     e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
@@ -372,7 +379,8 @@ def run_ours(args, rank, world, local_rank):
         "data": "synthetic (seeded): X ~ N(0, 0.02^2) fp32, P = 0 fp32, grad ~ N(0, 1e-3^2) bf16",
         "config": {"workload": desc, "params": N, "tensors": len(shapes), "matrices": mats,
                    "vector_elements": one_d, "grad_dtype": "bf16", "state_dtype": "f32",
-                   "hyperparameters": dict(HP, h=STEP),
+                   "hyperparameters": dict(hp, h=STEP), "method": args.method,
+                   "step_size": "alternating %g / %g" % hs if args.vary_h else "constant",
                    "l2": "no flush: %.2f GB of inputs per step > 129 MB L2" % (alg_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "hbm_gbs_step": round(alg_bytes / (ms_per_step / 1e3) / 1e9, 1),
@@ -385,10 +393,10 @@ def run_ours(args, rank, world, local_rank):
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": clocks,
-        "state_bytes": {"rikfad": state, "full_friction_ikfad": full_state,
+        "state_bytes": {args.method: state, "full_friction_ikfad": full_state,
                         "ratio": round(full_state / state, 3)},
     }
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and args.method == "rikfad":
         line["cpu_baseline"] = cpu_baseline(named, seed)
     return line
 
@@ -427,6 +435,12 @@ def main():
     ap.add_argument("--workload", default="gpt2s",
                     help="gpt2s (default), nano, sweep0..sweep3")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--method", choices=("rikfad", "ikfad"), default="rikfad",
+                    help="rikfad (default) or full-friction ikfad for comparison")
+    ap.add_argument("--gamma", type=float, default=HP["gamma"],
+                    help="linear damping gamma (default 0, R-iKFAD0)")
+    ap.add_argument("--vary-h", action="store_true",
+                    help="alternate the step size between h and 0.9 h")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")

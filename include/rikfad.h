@@ -99,6 +99,18 @@ typedef struct rikfad_handle_s *rikfad_handle;
 RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
                              int grad_dtype, rikfad_handle *out);
 
+/*
+ * Create a full-friction iKFAD optimiser (the method R-iKFAD factorises,
+ * Eqs. ikfad_1 to ikfad_3): every tensor, matrix or not, keeps one friction
+ * scalar per element and follows the element-wise rule; the auxiliary state
+ * is 2N floats (the iKFAD column of the paper's memory table).  Same handle
+ * type, step, checkpoint and query calls as rikfad_create; rikfad_get_factors
+ * returns a tensor's rows x cols friction values in R_host.  Every pointer
+ * must be 16-byte aligned.  Errors as for rikfad_create.
+ */
+RIKFAD_API int rikfad_create_ikfad(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
+                                   int grad_dtype, rikfad_handle *out);
+
 /* Release the handle and everything it allocated (after a device sync of its
  * own work).  NULL is accepted. */
 RIKFAD_API void rikfad_destroy(rikfad_handle h);

@@ -322,6 +322,9 @@ int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool 
     return RIKFAD_OK;
 }
 
+int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp, int grad_dtype,
+                rikfad_handle *out);
+
 }  // namespace
 
 extern "C" {
@@ -378,6 +381,35 @@ RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, i
 
 RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
                              int grad_dtype, rikfad_handle *out)
+{
+    return create_impl(shapes, ntensors, hp, grad_dtype, out);
+}
+
+RIKFAD_API int rikfad_create_ikfad(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
+                                   int grad_dtype, rikfad_handle *out)
+{
+    if (out == nullptr)
+        return fail(RIKFAD_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    std::string why = check_shapes(shapes, ntensors);
+    if (!why.empty())
+        return fail(RIKFAD_ERR_ARG, why);
+    // Full friction: every tensor follows the element-wise rule over its
+    // rows x cols elements.
+    std::vector<rikfad_shape> flat(ntensors);
+    for (int t = 0; t < ntensors; ++t) {
+        flat[t].rows = shapes[t].cols == 0 ? shapes[t].rows : shapes[t].rows * shapes[t].cols;
+        flat[t].cols = 0;
+    }
+    return create_impl(flat.data(), ntensors, hp, grad_dtype, out);
+}
+
+}  // extern "C"
+
+namespace {
+
+int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp, int grad_dtype,
+                rikfad_handle *out)
 {
     if (out == nullptr)
         return fail(RIKFAD_ERR_ARG, "out is NULL");
@@ -456,6 +488,10 @@ RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rik
     *out = h;
     return RIKFAD_OK;
 }
+
+}  // namespace
+
+extern "C" {
 
 RIKFAD_API void rikfad_destroy(rikfad_handle h)
 {

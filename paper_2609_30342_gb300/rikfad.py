@@ -47,6 +47,9 @@ _PP = ctypes.POINTER(ctypes.c_void_p)
 SIGNATURES = [
     ("rikfad_create", ctypes.c_int, [ctypes.POINTER(Shape), ctypes.c_int, ctypes.POINTER(HParams),
                                      ctypes.c_int, ctypes.POINTER(_VP)]),
+    ("rikfad_create_ikfad", ctypes.c_int, [ctypes.POINTER(Shape), ctypes.c_int,
+                                           ctypes.POINTER(HParams), ctypes.c_int,
+                                           ctypes.POINTER(_VP)]),
     ("rikfad_destroy", None, [_VP]),
     ("rikfad_step", ctypes.c_int, [_VP, ctypes.c_double, _PP, _PP, _PP, _VP]),
     ("rikfad_materialize", ctypes.c_int, [_VP, _PP, _VP]),
@@ -177,16 +180,23 @@ class RIKFAD:
     ``shapes``: list of ``(rows, cols)``; ``cols == 0`` marks a tensor that is
     not a matrix (``rows`` elements, element-wise rule).  Hyperparameters as
     in the paper (Section 2): ``alpha`` factor decay, ``mu`` friction scale,
-    ``gamma`` linear damping, ``eps_stab`` stabiliser.
+    ``gamma`` linear damping, ``eps_stab`` stabiliser.  ``method="ikfad"``
+    creates full-friction iKFAD instead (element-wise friction on every
+    tensor, ``rikfad_create_ikfad``).
     """
 
-    def __init__(self, shapes, alpha, mu, gamma=0.0, eps_stab=1e-16, grad_dtype="bf16"):
+    def __init__(self, shapes, alpha, mu, gamma=0.0, eps_stab=1e-16, grad_dtype="bf16",
+                 method="rikfad"):
+        if method not in ("rikfad", "ikfad"):
+            raise ValueError("method must be 'rikfad' or 'ikfad'")
+        self.method = method
         self.shapes = [(int(m), int(n)) for m, n in shapes]
         self.grad_dtype = GRAD_BF16 if grad_dtype in ("bf16", GRAD_BF16) else GRAD_F32
         hp = HParams(float(alpha), float(mu), float(gamma), float(eps_stab))
         h = ctypes.c_void_p()
-        _check(lib().rikfad_create(_shapes(self.shapes), len(self.shapes), ctypes.byref(hp),
-                                   self.grad_dtype, ctypes.byref(h)))
+        create = lib().rikfad_create if method == "rikfad" else lib().rikfad_create_ikfad
+        _check(create(_shapes(self.shapes), len(self.shapes), ctypes.byref(hp), self.grad_dtype,
+                      ctypes.byref(h)))
         self._h = h
 
     @property
@@ -237,8 +247,13 @@ class RIKFAD:
         return lib().rikfad_pending_step(self.handle)
 
     def get_factors(self, t):
-        """(R, C) of matrix t, or (friction, None) of a vector, as float32 numpy."""
+        """(R, C) of matrix t, or (friction, None) of a vector (of every tensor,
+        flattened, under full-friction iKFAD), as float32 numpy."""
+        if not 0 <= t < len(self.shapes):
+            raise RikfadError(ERR_ARG, "tensor index %d out of range" % t)
         m, n = self.shapes[t]
+        if self.method == "ikfad":
+            m, n = (m if n == 0 else m * n), 0
         R = np.zeros(m, np.float32)
         C = np.zeros(n, np.float32) if n else None
         _check(lib().rikfad_get_factors(self.handle, int(t), R.ctypes.data if m else None,

@@ -48,11 +48,11 @@ def compare(name, gpu, ref, rtol, floor):
 class GpuRun:
     """R-iKFAD on the GPU through the C ABI, with host-side inputs."""
 
-    def __init__(self, shapes, hp, grad_bf16, X, P, device="cuda"):
+    def __init__(self, shapes, hp, grad_bf16, X, P, device="cuda", method="rikfad"):
         self.shapes = [tuple(s) for s in shapes]
         self.grad_bf16 = grad_bf16
         self.opt = rikfad.RIKFAD(self.shapes, hp.alpha, hp.mu, hp.gamma, hp.eps_stab,
-                                 "bf16" if grad_bf16 else "f32")
+                                 "bf16" if grad_bf16 else "f32", method=method)
         gdt = torch.bfloat16 if grad_bf16 else torch.float32
         self.x = [torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device) for a in X]
         self.p = [torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device) for a in P]
