@@ -4,12 +4,14 @@
 
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
 
 #include "rikfad.h"
 #include "rikfad_aux_kernels.cuh"
+#include "rikfad_sweep.cuh"
 #include "rikfad_planner.hpp"
 
 using namespace rikfad;
@@ -97,6 +99,16 @@ struct rikfad_handle_s {
 
     PtrTable step_ptrs;             // x | grad | p
     PtrTable canon_ptrs;            // src | dst
+
+    // in-order ("sweep") schedule
+    bool sweep = true;
+    int sweep_blocks = 0;
+    UnitDev *d_units = nullptr;
+    NodeDev *d_nodes = nullptr;
+    PanelTreeDev *d_trees = nullptr;
+    float *d_partials = nullptr;
+    int32_t *d_counts = nullptr;    // node counters | tensor counters
+    unsigned long long *d_fetch = nullptr;   // unit counter | exit counter
 
     bool profiling = false;
     std::vector<cudaEvent_t> prof_events;   // 3 per recorded step
@@ -230,6 +242,12 @@ void release(rikfad_handle h)
     cudaFree(h->d_colpart);
     cudaFree(h->d_spart);
     cudaFree(h->d_den);
+    cudaFree(h->d_units);
+    cudaFree(h->d_nodes);
+    cudaFree(h->d_trees);
+    cudaFree(h->d_partials);
+    cudaFree(h->d_counts);
+    cudaFree(h->d_fetch);
     if (h->h_den)
         cudaFreeHost(h->h_den);
     ptrtable_free(h->step_ptrs);
@@ -257,6 +275,15 @@ void launch_step(const StepParams &p, bool reuse, int nblocks, cudaStream_t s)
         rikfad_step_kernel<GT, true><<<nblocks, kThreads, 0, s>>>(p);
     else
         rikfad_step_kernel<GT, false><<<nblocks, kThreads, 0, s>>>(p);
+}
+
+template <typename GT>
+void launch_sweep(const StepParams &p, const SweepParams &sp, bool reuse, int nblocks, cudaStream_t s)
+{
+    if (reuse)
+        rikfad_sweep_kernel<GT, true><<<nblocks, kThreads, 0, s>>>(p, sp);
+    else
+        rikfad_sweep_kernel<GT, false><<<nblocks, kThreads, 0, s>>>(p, sp);
 }
 
 int finalize(rikfad_handle h, float decay, float gain, int resum_only, cudaStream_t stream)
@@ -441,6 +468,18 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     }
     if (occ_min < 1)
         return fail(RIKFAD_ERR_CUDA, "step kernel cannot be resident on this device");
+    int occ_sweep = 1 << 30;
+    const void *sweep_kernels[4] = {(const void *)rikfad_sweep_kernel<float, true>,
+                                    (const void *)rikfad_sweep_kernel<float, false>,
+                                    (const void *)rikfad_sweep_kernel<__nv_bfloat16, true>,
+                                    (const void *)rikfad_sweep_kernel<__nv_bfloat16, false>};
+    for (const void *k : sweep_kernels) {
+        RK_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, 0),
+                "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+        occ_sweep = std::min(occ_sweep, occ);
+    }
+    if (occ_sweep < 1)
+        return fail(RIKFAD_ERR_CUDA, "sweep kernel cannot be resident on this device");
 
     rikfad_handle h = new rikfad_handle_s();
     h->device = dev;
@@ -454,6 +493,14 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
         delete h;
         return fail(RIKFAD_ERR_ARG, why);
     }
+    build_sweep(shapes, ntensors, h->plan);
+    {
+        // Static schedule by default; RIKFAD_SCHEDULE=sweep selects the
+        // in-order one-kernel schedule (slower on GB300, see rikfad_sweep.cuh).
+        const char *env = std::getenv("RIKFAD_SCHEDULE");
+        h->sweep = env && std::strcmp(env, "sweep") == 0;
+    }
+    h->sweep_blocks = sms * occ_sweep;
     const Plan &p = h->plan;
     size_t ws = 0;
     int rc = RIKFAD_OK;
@@ -471,6 +518,12 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     if (!rc) rc = alloc_zero(&h->d_den, std::max(ntensors, 1), ws);
     if (!rc && cudaMallocHost((void **)&h->h_den, sizeof(float) * std::max(ntensors, 1)) != cudaSuccess)
         rc = fail(RIKFAD_ERR_OOM, "cudaMallocHost failed");
+    if (!rc) rc = upload(&h->d_units, p.units, ws);
+    if (!rc) rc = upload(&h->d_nodes, p.nodes, ws);
+    if (!rc) rc = upload(&h->d_trees, p.trees, ws);
+    if (!rc) rc = alloc_zero(&h->d_partials, p.partial_floats, ws);
+    if (!rc) rc = alloc_zero((float **)&h->d_counts, (int64_t)p.nodes.size() + ntensors + 1, ws);
+    if (!rc) rc = alloc_zero((float **)&h->d_fetch, 4, ws);
     if (!rc) rc = ptrtable_init(h->step_ptrs, 3 * ntensors, ws);
     if (!rc) rc = ptrtable_init(h->canon_ptrs, 2 * ntensors, ws);
     if (!rc) {
@@ -560,7 +613,11 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
         h->prof_used += 3;
         RK_CUDA(cudaEventRecord(ev[0], s), "cudaEventRecord");
     }
-    if (h->plan.nblocks > 0) {
+    // Static schedule: the step kernel (if any element) then the finalise
+    // kernel.  Sweep schedule: one kernel does both (it also runs when only
+    // matrices without rows are present: their C still decays).
+    const bool run_kernel = h->sweep ? !h->plan.units.empty() : h->plan.nblocks > 0;
+    if (run_kernel) {
         StepParams a{};
         a.tensors = h->d_tensors;
         a.panels = h->d_panels;
@@ -582,17 +639,38 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
         a.gain = (float)gain_d;
         a.eps = (float)h->hp.eps_stab;
         const bool reuse = (step == h->pending_step);
-        if (h->grad_bytes == 2)
-            launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s);
-        else
-            launch_step<float>(a, reuse, h->plan.nblocks, s);
-        RK_CUDA(cudaGetLastError(), "launch rikfad_step_kernel");
+        if (h->sweep) {
+            SweepParams sp{};
+            sp.units = h->d_units;
+            sp.nodes = h->d_nodes;
+            sp.trees = h->d_trees;
+            sp.nunits = (int64_t)h->plan.units.size();
+            sp.partials = h->d_partials;
+            sp.spart = h->d_spart;
+            sp.node_count = h->d_counts;
+            sp.tensor_count = h->d_counts + h->plan.nodes.size();
+            sp.fetch = h->d_fetch;
+            sp.exits = reinterpret_cast<unsigned int *>(h->d_fetch + 1);
+            if (h->grad_bytes == 2)
+                launch_sweep<__nv_bfloat16>(a, sp, reuse, h->sweep_blocks, s);
+            else
+                launch_sweep<float>(a, sp, reuse, h->sweep_blocks, s);
+            RK_CUDA(cudaGetLastError(), "launch rikfad_sweep_kernel");
+        } else {
+            if (h->grad_bytes == 2)
+                launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s);
+            else
+                launch_step<float>(a, reuse, h->plan.nblocks, s);
+            RK_CUDA(cudaGetLastError(), "launch rikfad_step_kernel");
+        }
     }
     if (ev)
         RK_CUDA(cudaEventRecord(ev[1], s), "cudaEventRecord");
-    rc = finalize(h, (float)decay_d, (float)gain_d, 0, s);
-    if (rc)
-        return rc;
+    if (!h->sweep) {
+        rc = finalize(h, (float)decay_d, (float)gain_d, 0, s);
+        if (rc)
+            return rc;
+    }
     if (ev)
         RK_CUDA(cudaEventRecord(ev[2], s), "cudaEventRecord");
     h->pending_step = step;
@@ -805,6 +883,8 @@ RIKFAD_API int rikfad_launches_per_step(rikfad_handle h)
 {
     if (h == nullptr)
         return 0;
+    if (h->sweep)
+        return h->plan.units.empty() ? 0 : 1;
     return (h->plan.nblocks > 0 ? 1 : 0) + (h->plan.fin_items.empty() ? 0 : 1);
 }
 

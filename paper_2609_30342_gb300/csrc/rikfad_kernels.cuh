@@ -154,7 +154,9 @@ __device__ __forceinline__ float matrix_element(float &x, float p_hat, float g, 
 #define RIKFAD_CHUNK_GROUP 1
 #endif
 
-template <typename GT, bool REUSE>
+// ACCUM: add each row's squares into the warp's column buffer (several rows
+// per warp); otherwise store them (one row per warp, buffer not cleared).
+template <typename GT, bool REUSE, bool ACCUM = true>
 __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const PieceDev &pc,
                                                  const TensorDev &td, const PanelDev &pd,
                                                  const float *Cs, float *red, float inv)
@@ -212,11 +214,16 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
                     store8(X + base + c, xv[k]);
                     store8(P + base + c, pv[k]);
                     float4 *r4 = reinterpret_cast<float4 *>(myred + c);
-                    float4 r0 = r4[0], r1 = r4[1];
-                    r0.x += q[0]; r0.y += q[1]; r0.z += q[2]; r0.w += q[3];
-                    r1.x += q[4]; r1.y += q[5]; r1.z += q[6]; r1.w += q[7];
-                    r4[0] = r0;
-                    r4[1] = r1;
+                    if (ACCUM) {
+                        float4 r0 = r4[0], r1 = r4[1];
+                        r0.x += q[0]; r0.y += q[1]; r0.z += q[2]; r0.w += q[3];
+                        r1.x += q[4]; r1.y += q[5]; r1.z += q[6]; r1.w += q[7];
+                        r4[0] = r0;
+                        r4[1] = r1;
+                    } else {
+                        r4[0] = make_float4(q[0], q[1], q[2], q[3]);
+                        r4[1] = make_float4(q[4], q[5], q[6], q[7]);
+                    }
                 }
             }
         }
@@ -229,7 +236,7 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
 // ----------------------------------------------- matrix piece, scalar
 // For matrices whose rows are not 8-aligned (cols % 8 != 0).
 
-template <typename GT, bool REUSE>
+template <typename GT, bool REUSE, bool ACCUM = true>
 __device__ __forceinline__ void matrix_piece_scalar(const StepParams &a, const PieceDev &pc,
                                                     const TensorDev &td, const PanelDev &pd,
                                                     const float *Cs, float *red, float inv)
@@ -259,7 +266,10 @@ __device__ __forceinline__ void matrix_piece_scalar(const StepParams &a, const P
             P[base + c] = p1;
             const float q = p1 * p1;
             racc += q;
-            myred[c] += q;
+            if (ACCUM)
+                myred[c] += q;
+            else
+                myred[c] = q;
         }
         racc = warp_sum(racc);
         if (lane == 0)

@@ -71,4 +71,44 @@ struct FinItemDev {
     int64_t end;
 };
 
+// ------------------------------------------------------------------------
+// In-order schedule ("sweep"): persistent blocks take small units of work
+// from a global counter in memory order, so the whole GPU streams through a
+// narrow window of HBM at a time.  A matrix unit is up to kUnitRows rows of
+// one panel (one row per warp); a vector unit is up to kUnitElems elements.
+// Column partial sums of the units of a panel are combined up a static
+// kTreeFan-ary tree, in fixed order, by the block that completes a node's
+// last child; the block that completes a tensor's last panel updates R, C
+// and the partial sums of R in the same launch.
+constexpr int kUnitRows = kWarps;        // 8
+constexpr int64_t kUnitElems = 4096;
+constexpr int kTreeFan = 16;
+
+enum UnitKind : int32_t { kUnitMatrix = 0, kUnitVector = 1, kUnitFactorsOnly = 2 };
+
+struct UnitDev {
+    int32_t kind;
+    int32_t tensor;
+    int32_t panel;        // matrix units
+    int32_t parent;       // matrix units: tree node that combines this unit's partial
+    int64_t begin;        // first row (matrix) or element (vector)
+    int64_t end;
+    int64_t leaf_off;     // matrix units: float offset of this unit's column partial
+};
+
+struct NodeDev {
+    int32_t nchildren;
+    int32_t parent;       // -1: root of its panel
+    int32_t panel;
+    int32_t pad_;
+    int64_t first_child_off;  // children's partials are contiguous, PanelTreeDev::slot floats apart
+    int64_t off;              // this node's partial
+};
+
+struct PanelTreeDev {
+    int32_t slot;         // floats between consecutive partials of this panel (width rounded up to 32)
+    int32_t pad_;
+    int64_t root_off;     // partial of the panel's root node (column sums of the whole panel)
+};
+
 }  // namespace rikfad

@@ -210,4 +210,105 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
     return "";
 }
 
+void build_sweep(const rikfad_shape *shapes, int ntensors, Plan &plan)
+{
+    Plan &p = plan;
+    p.units.clear();
+    p.nodes.clear();
+    p.trees.assign(p.panels.size(), PanelTreeDev{});
+    int64_t off = 0;
+    for (int t = 0; t < ntensors; ++t) {
+        const TensorDev &td = p.tensors[t];
+        if (td.cols == 0)
+            continue;
+        if (td.rows == 0) {
+            UnitDev u{};
+            u.kind = kUnitFactorsOnly;
+            u.tensor = t;
+            u.panel = -1;
+            u.parent = -1;
+            p.units.push_back(u);
+            continue;
+        }
+        const int64_t first_unit = (int64_t)p.units.size();
+        const int64_t nrb = ceil_div(td.rows, kUnitRows);
+        // Units in memory order: row block major, panel minor.
+        for (int64_t rb = 0; rb < nrb; ++rb)
+            for (int32_t k = 0; k < td.npanels; ++k) {
+                UnitDev u{};
+                u.kind = kUnitMatrix;
+                u.tensor = t;
+                u.panel = td.panel0 + k;
+                u.begin = rb * kUnitRows;
+                u.end = std::min<int64_t>(td.rows, u.begin + kUnitRows);
+                p.units.push_back(u);
+            }
+        // One tree per panel over its nrb units.
+        for (int32_t k = 0; k < td.npanels; ++k) {
+            const int32_t panel = td.panel0 + k;
+            const int64_t slot = round_up(p.panels[panel].width, 32);
+            PanelTreeDev &tr = p.trees[panel];
+            tr.slot = (int32_t)slot;
+            // leaves: the panel's units, in row order
+            const int64_t leaf0 = off;
+            for (int64_t rb = 0; rb < nrb; ++rb) {
+                UnitDev &u = p.units[first_unit + rb * td.npanels + k];
+                u.leaf_off = leaf0 + rb * slot;
+            }
+            off += nrb * slot;
+            // internal levels until one node remains (a single leaf still gets a root)
+            int64_t count = nrb, child_off = leaf0;
+            std::vector<int32_t> child_ids;      // node ids of the previous level (empty: leaves)
+            for (;;) {
+                const int64_t nn = ceil_div(count, kTreeFan);
+                const int64_t level_off = off;
+                std::vector<int32_t> ids;
+                for (int64_t j = 0; j < nn; ++j) {
+                    NodeDev nd{};
+                    nd.nchildren = (int32_t)std::min<int64_t>(kTreeFan, count - j * kTreeFan);
+                    nd.parent = -1;
+                    nd.panel = panel;
+                    nd.first_child_off = child_off + j * kTreeFan * slot;
+                    nd.off = level_off + j * slot;
+                    const int32_t id = (int32_t)p.nodes.size();
+                    p.nodes.push_back(nd);
+                    ids.push_back(id);
+                    for (int64_t c = j * kTreeFan; c < j * kTreeFan + nd.nchildren; ++c) {
+                        if (child_ids.empty())
+                            p.units[first_unit + c * td.npanels + k].parent = id;
+                        else
+                            p.nodes[child_ids[c]].parent = id;
+                    }
+                }
+                off += nn * slot;
+                if (nn == 1) {
+                    tr.root_off = p.nodes[ids[0]].off;
+                    break;
+                }
+                child_ids = ids;
+                child_off = level_off;
+                count = nn;
+            }
+        }
+    }
+    // vectors last
+    for (int t = 0; t < ntensors; ++t) {
+        const TensorDev &td = p.tensors[t];
+        if (td.cols != 0)
+            continue;
+        for (int64_t b = 0; b < td.rows; b += kUnitElems) {
+            UnitDev u{};
+            u.kind = kUnitVector;
+            u.tensor = t;
+            u.panel = -1;
+            u.parent = -1;
+            u.begin = b;
+            u.end = std::min<int64_t>(td.rows, b + kUnitElems);
+            p.units.push_back(u);
+        }
+    }
+    p.partial_floats = off;
+    (void)shapes;
+}
+
 }  // namespace rikfad

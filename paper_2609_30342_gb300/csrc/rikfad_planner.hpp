@@ -21,7 +21,17 @@ struct Plan {
     int32_t spart_floats = 0;
     int nblocks = 0;                    // blocks of the step kernel (0 when there is no work)
     int64_t total_bytes = 0;            // compulsory HBM bytes of one step (planner's cost model)
+
+    // In-order schedule (see rikfad_plan.hpp)
+    std::vector<UnitDev> units;
+    std::vector<NodeDev> nodes;
+    std::vector<PanelTreeDev> trees;    // one per panel
+    int64_t partial_floats = 0;         // unit and node partials
 };
+
+// Add the in-order schedule (units, reduction trees) to a plan built by
+// build_plan.  Matrices keep their order; vectors come last.
+void build_sweep(const rikfad_shape *shapes, int ntensors, Plan &plan);
 
 // Validate the shape list; returns "" or an error message.
 std::string check_shapes(const rikfad_shape *shapes, int ntensors);

@@ -240,7 +240,8 @@ def test_profile_counters():
     for _ in range(5):
         run.step(0.1)
     a, b, n = run.opt.profile_read()
-    assert n == 5 and a > 0 and b > 0
-    assert run.opt.launches_per_step() == 2
+    assert n == 5 and a > 0 and b >= 0
+    # one kernel per step with the in-order schedule, step + finalise otherwise
+    assert run.opt.launches_per_step() in (1, 2)
     run.opt.profile_enable(False)
     run.close()
