@@ -268,13 +268,31 @@ bool aligned_for(const TensorDev &td, const void *ptr, size_t natural)
 
 int64_t numel(const TensorDev &td) { return td.cols == 0 ? td.rows : td.rows * td.cols; }
 
+// Launch with programmatic stream serialisation: the kernel may begin while
+// its predecessor in the stream finishes; it waits (griddepcontrol.wait)
+// before touching any data.
+template <typename Kern, typename Arg>
+cudaError_t launch_pdl(Kern kernel, int nblocks, int nthreads, cudaStream_t s, const Arg &arg)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)nblocks);
+    cfg.blockDim = dim3((unsigned)nthreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, arg);
+}
+
 template <typename GT>
-void launch_step(const StepParams &p, bool reuse, int nblocks, cudaStream_t s)
+cudaError_t launch_step(const StepParams &p, bool reuse, int nblocks, cudaStream_t s)
 {
     if (reuse)
-        rikfad_step_kernel<GT, true><<<nblocks, kThreads, 0, s>>>(p);
-    else
-        rikfad_step_kernel<GT, false><<<nblocks, kThreads, 0, s>>>(p);
+        return launch_pdl(rikfad_step_kernel<GT, true>, nblocks, kThreads, s, p);
+    return launch_pdl(rikfad_step_kernel<GT, false>, nblocks, kThreads, s, p);
 }
 
 template <typename GT>
@@ -302,8 +320,8 @@ int finalize(rikfad_handle h, float decay, float gain, int resum_only, cudaStrea
     f.decay = decay;
     f.gain = gain;
     f.resum_only = resum_only;
-    rikfad_finalize_kernel<<<(unsigned)h->plan.fin_items.size(), kFinThreads, 0, stream>>>(f);
-    RK_CUDA(cudaGetLastError(), "launch rikfad_finalize_kernel");
+    RK_CUDA(launch_pdl(rikfad_finalize_kernel, (int)h->plan.fin_items.size(), kFinThreads, stream, f),
+            "launch rikfad_finalize_kernel");
     return RIKFAD_OK;
 }
 
@@ -658,10 +676,9 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
             RK_CUDA(cudaGetLastError(), "launch rikfad_sweep_kernel");
         } else {
             if (h->grad_bytes == 2)
-                launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s);
+                RK_CUDA(launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s), "launch rikfad_step_kernel");
             else
-                launch_step<float>(a, reuse, h->plan.nblocks, s);
-            RK_CUDA(cudaGetLastError(), "launch rikfad_step_kernel");
+                RK_CUDA(launch_step<float>(a, reuse, h->plan.nblocks, s), "launch rikfad_step_kernel");
         }
     }
     if (ev)

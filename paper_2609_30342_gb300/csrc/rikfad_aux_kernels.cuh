@@ -48,16 +48,20 @@ struct FinParams {
 // C_{n+1} = e^{-alpha h} C_n + k sum_slots colpart,
 // and the partial sums of R_{n+1} that give 1^T R_{n+1}.
 //
-// A row item is kFinThreads rows, one thread per row.  A column item is
-// kFinColChunk (32) columns of one panel: warp w adds the slots
-// slot_begin + w, + 8, ... for the 32 columns (coalesced 128-byte rows of the
-// partials), then warp 0 adds the eight warp sums in order.
+// A row item is kFinThreads rows, one thread per row.  A column item of a
+// panel with few slots is up to 256 columns, one thread per column adding the
+// slots in order; a panel with many slots (more than kFinSplitSlots) gets
+// items of kFinColChunk (32) columns: warp w adds the slots slot_begin + w,
+// + 8, ... for the 32 columns (coalesced 128-byte rows of the partials), then
+// warp 0 adds the eight warp sums in order.
 __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams f)
 {
     __shared__ float wsum[kFinThreads / 32];
     __shared__ float csum[kFinThreads / 32][32];
     const FinItemDev it = f.items[blockIdx.x];
     const TensorDev td = f.tensors[it.tensor];
+    wait_for_predecessor();
+    allow_successor_launch();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (it.kind == kFinRows) {
         const int64_t i = it.begin + threadIdx.x;
@@ -84,6 +88,16 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
             v = warp_sum(v);
             if (threadIdx.x == 0)
                 f.spart[td.spart_off + it.chunk] = v;
+        }
+    } else if (!f.resum_only && it.chunk == 0) {
+        const PanelDev pd = f.panels[it.panel];
+        const int64_t c = it.begin + threadIdx.x;
+        if (c < it.end) {
+            float acc = 0.f;
+            for (int s = pd.slot_begin; s < pd.slot_end; ++s)
+                acc += f.colpart[f.slot_off[s] + c];
+            float *C = f.fac + td.fac_off + td.rows + pd.col0;
+            C[c] = fmaf(f.gain, acc, f.decay * C[c]);
         }
     } else if (!f.resum_only) {
         const PanelDev pd = f.panels[it.panel];

@@ -55,6 +55,20 @@ struct StepParams {
 
 // ---------------------------------------------------------------- helpers
 
+// Programmatic dependent launch: the kernels of a step are launched so that
+// they may start before their predecessor in the stream has finished; they
+// run this wait before touching any data the predecessor may write, and let
+// their own successor start launching early.
+__device__ __forceinline__ void wait_for_predecessor()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+__device__ __forceinline__ void allow_successor_launch()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ float warp_sum(float v)
 {
     // Butterfly: float addition is commutative, so every lane ends with the
@@ -340,6 +354,8 @@ __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_
     __shared__ __align__(16) float red[kWarps * kPanelMax];
     const int b = blockIdx.x;
     const int q0 = a.block_piece[b], q1 = a.block_piece[b + 1];
+    wait_for_predecessor();
+    allow_successor_launch();
     for (int q = q0; q < q1; ++q) {
         const PieceDev pc = a.pieces[q];
         const TensorDev td = a.tensors[pc.tensor];

@@ -22,7 +22,8 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kPanelMax = 1024;      // widest column panel (floats staged in shared memory)
 constexpr int kChunk = 256;          // columns one warp covers per pass (32 lanes x 8)
 constexpr int kFinThreads = 256;     // threads of the finalise kernel (= rows per partial sum)
-constexpr int kFinColChunk = 32;     // columns per finalise column item
+constexpr int kFinColChunk = 32;     // columns per split column item (8 warps share its slots)
+constexpr int kFinSplitSlots = 8;    // panels with more slots than this get split column items
 constexpr int kElemGranule = 8;      // element pieces start on multiples of 8 elements
 constexpr int64_t kMinBlockBytes = 64 * 1024;   // smallest share worth a block
 
@@ -66,7 +67,8 @@ struct FinItemDev {
     int32_t kind;
     int32_t tensor;
     int32_t panel;        // kFinCols
-    int32_t chunk;        // kFinRows: index of the partial sum of R within the tensor
+    int32_t chunk;        // kFinRows: index of the partial sum of R within the tensor;
+                          // kFinCols: 1 = split item (warps share the slots), 0 = one thread per column
     int64_t begin;        // kFinRows: rows; kFinCols: columns relative to the panel
     int64_t end;
 };

@@ -194,14 +194,18 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
         }
         for (int32_t k = 0; k < td.npanels; ++k) {
             const PanelDev &pd = p.panels[td.panel0 + k];
-            for (int64_t c0 = 0; c0 < pd.width; c0 += kFinColChunk) {
+            // Many slots: 32-column items whose 8 warps split the slots; few
+            // slots: one thread per column, 256 columns per item.
+            const bool split = pd.slot_end - pd.slot_begin > kFinSplitSlots;
+            const int64_t step = split ? kFinColChunk : kFinThreads;
+            for (int64_t c0 = 0; c0 < pd.width; c0 += step) {
                 FinItemDev it{};
                 it.kind = kFinCols;
                 it.tensor = t;
                 it.panel = td.panel0 + k;
-                it.chunk = 0;
+                it.chunk = split ? 1 : 0;
                 it.begin = c0;
-                it.end = std::min<int64_t>(pd.width, c0 + kFinColChunk);
+                it.end = std::min<int64_t>(pd.width, c0 + step);
                 p.fin_items.push_back(it);
             }
         }
