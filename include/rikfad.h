@@ -118,7 +118,10 @@ RIKFAD_API void rikfad_destroy(rikfad_handle h);
 /*
  * Enqueue one R-iKFAD step of size `step` (> 0, finite) over every tensor.
  *   x[t]    device, float32, tensor t's parameters; updated to X_{n+1}
- *   grad[t] device, float32 or bfloat16 (per handle), grad f(X_n); read only
+ *   grad[t] float32 or bfloat16 (per handle), grad f(X_n); read only.  Device
+ *           memory, or page-locked host memory that the device can address
+ *           (e.g. from cudaHostAlloc): the kernel then reads the gradient
+ *           over the CPU-GPU link, with no separate copy
  *   p[t]    device, float32, tensor t's momentum in the library's stored form
  *           (below); updated
  * The three arrays are host arrays of `ntensors` device pointers, in the

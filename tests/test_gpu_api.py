@@ -245,3 +245,22 @@ def test_profile_counters():
     assert run.opt.launches_per_step() in (1, 2)
     run.opt.profile_enable(False)
     run.close()
+
+
+def test_pinned_host_gradients_read_in_place():
+    """Gradients may live in page-locked host memory: the step kernel reads
+    them across the CPU-GPU link and gives bitwise the same step."""
+    inp, run_d = _run()
+    _, run_h = _run()
+    g = inp.grads(0)
+    run_d.set_grads(g)
+    host_g = [torch.from_numpy(a).to(torch.bfloat16).pin_memory() for a in g]
+    ptr_h = run_h.opt.pack(run_h.x, host_g, run_h.p)
+    for h in (0.1, 0.1, 0.05):
+        run_d.step(h)
+        run_h.opt.step(h, ptrs=ptr_h)
+    torch.cuda.synchronize()
+    for a, b in zip(run_d.x + run_d.p, run_h.x + run_h.p):
+        assert torch.equal(a, b)
+    run_d.close()
+    run_h.close()
