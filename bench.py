@@ -73,7 +73,7 @@ def algorithmic_bytes(shapes, grad_bytes, method="rikfad"):
     full-friction iKFAD every element is a vector element."""
     from paper_2609_30342_gb300 import workloads as W
     N, _, _, one_d = W.count(shapes)
-    if method == "ikfad":
+    if method in ("ikfad", "ikfad_shadow"):
         return N * (grad_bytes + 24)
     return (N - one_d) * (grad_bytes + 16) + one_d * (grad_bytes + 24)
 
@@ -377,6 +377,26 @@ def run_ours(args, rank, world, local_rank):
            "d2h_bytes_per_step": 4 * len(shapes),
            "h2d_path": "step kernel loads the bf16 gradients from pinned host memory (zero-copy)"}
 
+    diag = None
+    if args.diagnostics and args.method == "ikfad_shadow":
+        # Per-layer comparison of the paper's Section 4.4 on the final state:
+        # error of the shadow rank-1 friction vs the Eckart-Young floor, and
+        # the stable rank of the element-wise friction.
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        rows = []
+        for t, (m, n) in enumerate(shapes):
+            if n and m:
+                rows.append(opt.friction_diagnostics(t, stream=stream))
+        dt = time.perf_counter() - t0
+        gaps = [100.0 * (r[0] - r[1]) for r in rows]
+        diag = {"layers": len(rows), "seconds": round(dt, 3),
+                "median_gap_pp": round(float(np.median(gaps)), 4),
+                "max_gap_pp": round(float(np.max(gaps)), 4),
+                "stable_rank_min_max": [round(min(r[2] for r in rows), 4),
+                                        round(max(r[2] for r in rows), 4)],
+                "mean_power_iterations": round(float(np.mean([r[5] for r in rows])), 1)}
+
     launches = opt.launches_per_step() * args.steps
     state = opt.state_bytes(True)
     full_state = 8 * N
@@ -410,6 +430,8 @@ def run_ours(args, rank, world, local_rank):
         "state_bytes": {args.method: state, "full_friction_ikfad": full_state,
                         "ratio": round(full_state / state, 3)},
     }
+    if diag is not None:
+        line["friction_diagnostics"] = diag
     if world == 1 and not args.no_cpu_baseline and args.method == "rikfad":
         line["cpu_baseline"] = cpu_baseline(named, seed)
     return line
@@ -449,8 +471,10 @@ def main():
     ap.add_argument("--workload", default="gpt2s",
                     help="gpt2s (default), nano, sweep0..sweep3")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--method", choices=("rikfad", "ikfad"), default="rikfad",
-                    help="rikfad (default) or full-friction ikfad for comparison")
+    ap.add_argument("--method", choices=("rikfad", "ikfad", "ikfad_shadow"), default="rikfad",
+                    help="rikfad (default), full-friction ikfad, or ikfad with shadow R-iKFAD factors")
+    ap.add_argument("--diagnostics", action="store_true",
+                    help="with --method ikfad_shadow: per-layer friction diagnostics after timing")
     ap.add_argument("--gamma", type=float, default=HP["gamma"],
                     help="linear damping gamma (default 0, R-iKFAD0)")
     ap.add_argument("--vary-h", action="store_true",

@@ -111,6 +111,21 @@ RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rik
 RIKFAD_API int rikfad_create_ikfad(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
                                    int grad_dtype, rikfad_handle *out);
 
+/*
+ * Create full iKFAD with R-iKFAD's factors carried along as shadows: every
+ * matrix keeps its element-wise friction xi (rows x cols floats) and steps by
+ * full iKFAD, while its R and C follow R-iKFAD's factor filter from the same
+ * half-damped momentum without being used in the update.  This is the set-up
+ * of the paper's Section 4.4 ("How close is xi~ to the best rank-1
+ * friction?"), read out by rikfad_friction_diagnostics.  Non-matrices follow
+ * the element-wise rule as usual.  Same step and query calls as
+ * rikfad_create; momenta are always canonical (no pending factor).  Every
+ * pointer of a matrix whose cols is a multiple of 8 must be 16-byte aligned.
+ */
+RIKFAD_API int rikfad_create_ikfad_shadow(const rikfad_shape *shapes, int ntensors,
+                                          const rikfad_hparams *hp, int grad_dtype,
+                                          rikfad_handle *out);
+
 /* Release the handle and everything it allocated (after a device sync of its
  * own work).  NULL is accepted. */
 RIKFAD_API void rikfad_destroy(rikfad_handle h);
@@ -187,6 +202,31 @@ RIKFAD_API int rikfad_get_factors(rikfad_handle h, int t, float *R_host, float *
 /* Overwrite tensor t's factors from the host (same layout as
  * rikfad_get_factors; values must be finite and >= 0).  Synchronises. */
 RIKFAD_API int rikfad_set_factors(rikfad_handle h, int t, const float *R_host, const float *C_host);
+
+/* Copy tensor t's element-wise friction to the host (synchronises): the
+ * rows floats of a non-matrix, or the rows x cols floats (row-major) of a
+ * matrix of a shadow handle.  RIKFAD_ERR_ARG for a matrix with rank-1
+ * friction (its state is R and C, rikfad_get_factors). */
+RIKFAD_API int rikfad_get_friction(rikfad_handle h, int t, float *xi_host);
+
+/*
+ * Friction diagnostics of matrix t of a shadow handle (rikfad_create_ikfad_
+ * shadow), after the work enqueued on `stream` (synchronises).  Writes six
+ * doubles to out (host):
+ *   out[0]  ||xi - xi~||_F / ||xi||_F, xi~ = R C^T / (1^T R + eps_stab) from
+ *           the shadow factors (the error of R-iKFAD's construction)
+ *   out[1]  sqrt(1 - sigma_1^2 / ||xi||_F^2), the smallest relative error of
+ *           any rank-1 approximation (Eckart-Young)
+ *   out[2]  ||xi||_F^2 / sigma_1^2, the stable rank of xi
+ *   out[3]  sigma_1, by power iteration on xi^T xi started from C, stopped
+ *           when the estimate of sigma_1^2 changes by at most tol (relative)
+ *           or after max_iters iterations
+ *   out[4]  ||xi||_F
+ *   out[5]  iterations used
+ * All zeros for an all-zero friction.  RIKFAD_ERR_STATE for other handles.
+ */
+RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters, double tol, double *out,
+                                           void *stream);
 
 /* Read the friction denominators 1^T R of every matrix (ntensors floats, 0 for
  * element-wise tensors) into host memory, enqueued on `stream`; the values

@@ -12,6 +12,7 @@
 #include "rikfad.h"
 #include "rikfad_aux_kernels.cuh"
 #include "rikfad_sweep.cuh"
+#include "rikfad_diag_kernels.cuh"
 #include "rikfad_planner.hpp"
 
 using namespace rikfad;
@@ -99,6 +100,11 @@ struct rikfad_handle_s {
 
     PtrTable step_ptrs;             // x | grad | p
     PtrTable canon_ptrs;            // src | dst
+
+    // full iKFAD with shadow R-iKFAD factors (friction diagnostics)
+    bool shadow = false;
+    float *d_diag_u = nullptr, *d_diag_v = nullptr, *d_diag_w = nullptr, *d_diag_wpart = nullptr;
+    double *d_diag_norms = nullptr;
 
     // in-order ("sweep") schedule
     bool sweep = true;
@@ -242,6 +248,11 @@ void release(rikfad_handle h)
     cudaFree(h->d_colpart);
     cudaFree(h->d_spart);
     cudaFree(h->d_den);
+    cudaFree(h->d_diag_u);
+    cudaFree(h->d_diag_v);
+    cudaFree(h->d_diag_w);
+    cudaFree(h->d_diag_wpart);
+    cudaFree(h->d_diag_norms);
     cudaFree(h->d_units);
     cudaFree(h->d_nodes);
     cudaFree(h->d_trees);
@@ -288,8 +299,10 @@ cudaError_t launch_pdl(Kern kernel, int nblocks, int nthreads, cudaStream_t s, c
 }
 
 template <typename GT>
-cudaError_t launch_step(const StepParams &p, bool reuse, int nblocks, cudaStream_t s)
+cudaError_t launch_step(const StepParams &p, bool reuse, bool shadow, int nblocks, cudaStream_t s)
 {
+    if (shadow)     // full-friction matrices: reuse never applies (no pending factor)
+        return launch_pdl(rikfad_step_kernel<GT, false, true>, nblocks, kThreads, s, p);
     if (reuse)
         return launch_pdl(rikfad_step_kernel<GT, true>, nblocks, kThreads, s, p);
     return launch_pdl(rikfad_step_kernel<GT, false>, nblocks, kThreads, s, p);
@@ -368,7 +381,7 @@ int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool 
 }
 
 int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp, int grad_dtype,
-                rikfad_handle *out);
+                rikfad_handle *out, bool shadow = false);
 
 }  // namespace
 
@@ -430,6 +443,12 @@ RIKFAD_API int rikfad_create(const rikfad_shape *shapes, int ntensors, const rik
     return create_impl(shapes, ntensors, hp, grad_dtype, out);
 }
 
+RIKFAD_API int rikfad_create_ikfad_shadow(const rikfad_shape *shapes, int ntensors,
+                                          const rikfad_hparams *hp, int grad_dtype, rikfad_handle *out)
+{
+    return create_impl(shapes, ntensors, hp, grad_dtype, out, true);
+}
+
 RIKFAD_API int rikfad_create_ikfad(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp,
                                    int grad_dtype, rikfad_handle *out)
 {
@@ -454,7 +473,7 @@ RIKFAD_API int rikfad_create_ikfad(const rikfad_shape *shapes, int ntensors, con
 namespace {
 
 int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *hp, int grad_dtype,
-                rikfad_handle *out)
+                rikfad_handle *out, bool shadow)
 {
     if (out == nullptr)
         return fail(RIKFAD_ERR_ARG, "out is NULL");
@@ -475,10 +494,12 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     RK_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
     // Persistent grid: as many blocks as can be resident at once.
     int occ_min = 1 << 30;
-    const void *kernels[4] = {(const void *)rikfad_step_kernel<float, true>,
+    const void *kernels[6] = {(const void *)rikfad_step_kernel<float, true>,
                               (const void *)rikfad_step_kernel<float, false>,
                               (const void *)rikfad_step_kernel<__nv_bfloat16, true>,
-                              (const void *)rikfad_step_kernel<__nv_bfloat16, false>};
+                              (const void *)rikfad_step_kernel<__nv_bfloat16, false>,
+                              (const void *)rikfad_step_kernel<float, false, true>,
+                              (const void *)rikfad_step_kernel<__nv_bfloat16, false, true>};
     for (const void *k : kernels) {
         RK_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, 0),
                 "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
@@ -506,7 +527,8 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     h->hp = *hp;
     h->shapes.assign(shapes, shapes + ntensors);
     h->max_blocks = sms * occ_min;
-    why = build_plan(shapes, ntensors, h->grad_bytes, h->max_blocks, h->plan);
+    h->shadow = shadow;
+    why = build_plan(shapes, ntensors, h->grad_bytes, h->max_blocks, h->plan, shadow);
     if (!why.empty()) {
         delete h;
         return fail(RIKFAD_ERR_ARG, why);
@@ -516,7 +538,7 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
         // Static schedule by default; RIKFAD_SCHEDULE=sweep selects the
         // in-order one-kernel schedule (slower on GB300, see rikfad_sweep.cuh).
         const char *env = std::getenv("RIKFAD_SCHEDULE");
-        h->sweep = env && std::strcmp(env, "sweep") == 0;
+        h->sweep = env && std::strcmp(env, "sweep") == 0 && !shadow;
     }
     h->sweep_blocks = sms * occ_sweep;
     const Plan &p = h->plan;
@@ -542,6 +564,20 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     if (!rc) rc = alloc_zero(&h->d_partials, p.partial_floats, ws);
     if (!rc) rc = alloc_zero((float **)&h->d_counts, (int64_t)p.nodes.size() + ntensors + 1, ws);
     if (!rc) rc = alloc_zero((float **)&h->d_fetch, 4, ws);
+    if (!rc && shadow) {
+        int64_t max_m = 1, max_n = 1, max_parts = 1;
+        for (const TensorDev &td : p.tensors)
+            if (td.cols > 0) {
+                max_m = std::max(max_m, td.rows);
+                max_n = std::max(max_n, td.cols);
+                max_parts = std::max<int64_t>(max_parts, (td.rows + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
+            }
+        rc = alloc_zero(&h->d_diag_u, max_m, ws);
+        if (!rc) rc = alloc_zero(&h->d_diag_v, max_n, ws);
+        if (!rc) rc = alloc_zero(&h->d_diag_w, max_n, ws);
+        if (!rc) rc = alloc_zero(&h->d_diag_wpart, max_parts * max_n, ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_diag_norms, 4 * ((max_m + kWarps - 1) / kWarps), ws);
+    }
     if (!rc) rc = ptrtable_init(h->step_ptrs, 3 * ntensors, ws);
     if (!rc) rc = ptrtable_init(h->canon_ptrs, 2 * ntensors, ws);
     if (!rc) {
@@ -676,9 +712,10 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
             RK_CUDA(cudaGetLastError(), "launch rikfad_sweep_kernel");
         } else {
             if (h->grad_bytes == 2)
-                RK_CUDA(launch_step<__nv_bfloat16>(a, reuse, h->plan.nblocks, s), "launch rikfad_step_kernel");
+                RK_CUDA(launch_step<__nv_bfloat16>(a, reuse, h->shadow, h->plan.nblocks, s),
+                        "launch rikfad_step_kernel");
             else
-                RK_CUDA(launch_step<float>(a, reuse, h->plan.nblocks, s), "launch rikfad_step_kernel");
+                RK_CUDA(launch_step<float>(a, reuse, h->shadow, h->plan.nblocks, s), "launch rikfad_step_kernel");
         }
     }
     if (ev)
@@ -719,7 +756,12 @@ RIKFAD_API size_t rikfad_state_bytes(rikfad_handle h, int include_momentum)
 {
     if (h == nullptr)
         return 0;
-    return rikfad_state_bytes_for(h->shapes.data(), h->ntensors, include_momentum);
+    size_t b = rikfad_state_bytes_for(h->shapes.data(), h->ntensors, include_momentum);
+    if (h->shadow)      // plus the element-wise friction of every matrix
+        for (const rikfad_shape &sh : h->shapes)
+            if (sh.cols > 0)
+                b += sizeof(float) * (size_t)(sh.rows * sh.cols);
+    return b;
 }
 
 RIKFAD_API size_t rikfad_workspace_bytes(rikfad_handle h) { return h ? h->workspace : 0; }
@@ -903,6 +945,131 @@ RIKFAD_API int rikfad_launches_per_step(rikfad_handle h)
     if (h->sweep)
         return h->plan.units.empty() ? 0 : 1;
     return (h->plan.nblocks > 0 ? 1 : 0) + (h->plan.fin_items.empty() ? 0 : 1);
+}
+
+RIKFAD_API int rikfad_get_friction(rikfad_handle h, int t, float *xi_host)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (t < 0 || t >= h->ntensors)
+        return fail(RIKFAD_ERR_ARG, "tensor index out of range");
+    const TensorDev &td = h->plan.tensors[t];
+    int64_t off, count;
+    if (td.cols == 0) {
+        off = td.fac_off;
+        count = td.rows;
+    } else if (td.full) {
+        off = td.xi_off;
+        count = td.rows * td.cols;
+    } else {
+        return fail(RIKFAD_ERR_ARG, "tensor " + std::to_string(t) + " has rank-1 friction (use rikfad_get_factors)");
+    }
+    if (count > 0 && xi_host == nullptr)
+        return fail(RIKFAD_ERR_ARG, "xi_host is NULL");
+    RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    if (count > 0)
+        RK_CUDA(cudaMemcpy(xi_host, h->d_fac + off, sizeof(float) * count, cudaMemcpyDeviceToHost),
+                "cudaMemcpy friction");
+    return RIKFAD_OK;
+}
+
+RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters, double tol, double *out,
+                                           void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (!h->shadow)
+        return fail(RIKFAD_ERR_STATE, "friction diagnostics need a handle from rikfad_create_ikfad_shadow");
+    if (t < 0 || t >= h->ntensors || h->plan.tensors[t].cols == 0)
+        return fail(RIKFAD_ERR_ARG, "tensor index is not a matrix");
+    if (out == nullptr || max_iters < 1 || !(tol >= 0))
+        return fail(RIKFAD_ERR_ARG, "out is NULL, max_iters < 1 or tol < 0");
+    const TensorDev &td = h->plan.tensors[t];
+    const int64_t m = td.rows, n = td.cols;
+    for (int k = 0; k < 6; ++k)
+        out[k] = 0.0;
+    if (m == 0)
+        return RIKFAD_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    const float *xi = h->d_fac + td.xi_off;
+    const float *R = h->d_fac + td.fac_off;
+    const float *C = h->d_fac + td.fac_off + m;
+    // 1^T R exactly as the step kernels form it
+    DenParams d{h->d_tensors, h->d_spart, h->d_den, h->ntensors};
+    rikfad_denominators_kernel<<<(h->ntensors + kWarps - 1) / kWarps, kThreads, 0, s>>>(d);
+    RK_CUDA(cudaGetLastError(), "launch rikfad_denominators_kernel");
+    float den_sum = 0.f;
+    RK_CUDA(cudaMemcpyAsync(&den_sum, h->d_den + t, sizeof(float), cudaMemcpyDeviceToHost, s), "cudaMemcpyAsync");
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    const float den = den_sum + (float)h->hp.eps_stab;
+    const float inv = den == 0.f ? 0.f : 1.f / den;
+    // ||xi||^2 and ||xi - xi~||^2
+    const int nb_rows = (int)((m + kWarps - 1) / kWarps);
+    rikfad_diag_norms_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, R, C, inv, h->d_diag_norms);
+    RK_CUDA(cudaGetLastError(), "launch rikfad_diag_norms_kernel");
+    std::vector<double> parts(2 * (size_t)nb_rows);
+    RK_CUDA(cudaMemcpyAsync(parts.data(), h->d_diag_norms, sizeof(double) * parts.size(), cudaMemcpyDeviceToHost, s),
+            "cudaMemcpyAsync");
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    double f2 = 0.0, e2 = 0.0;
+    for (int b = 0; b < nb_rows; ++b) {
+        f2 += parts[2 * b];
+        e2 += parts[2 * b + 1];
+    }
+    // sigma_1 by power iteration on xi^T xi, starting from C (the shadow
+    // column factor, close to the top right singular vector).
+    std::vector<float> v(n), hw(n), hu(m);
+    RK_CUDA(cudaMemcpyAsync(v.data(), C, sizeof(float) * n, cudaMemcpyDeviceToHost, s), "cudaMemcpyAsync");
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    double vn = 0.0;
+    for (float x : v)
+        vn += (double)x * x;
+    vn = std::sqrt(vn);
+    for (int64_t j = 0; j < n; ++j)
+        v[j] = vn > 0 ? (float)(v[j] / vn) : (float)(1.0 / std::sqrt((double)n));
+    const int nb_t = (int)((m + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
+    double sigma2 = 0.0;
+    int it = 0;
+    for (it = 1; it <= max_iters; ++it) {
+        RK_CUDA(cudaMemcpyAsync(h->d_diag_v, v.data(), sizeof(float) * n, cudaMemcpyHostToDevice, s),
+                "cudaMemcpyAsync");
+        rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, h->d_diag_v, h->d_diag_u);
+        rikfad_diag_matvec_t_kernel<<<nb_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart);
+        rikfad_diag_colsum_kernel<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
+            h->d_diag_wpart, nb_t, n, h->d_diag_w);
+        RK_CUDA(cudaGetLastError(), "launch diagnostic kernels");
+        RK_CUDA(cudaMemcpyAsync(hu.data(), h->d_diag_u, sizeof(float) * m, cudaMemcpyDeviceToHost, s),
+                "cudaMemcpyAsync");
+        RK_CUDA(cudaMemcpyAsync(hw.data(), h->d_diag_w, sizeof(float) * n, cudaMemcpyDeviceToHost, s),
+                "cudaMemcpyAsync");
+        RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+        double u2 = 0.0, w2 = 0.0;
+        for (float x : hu)
+            u2 += (double)x * x;
+        for (float x : hw)
+            w2 += (double)x * x;
+        const double prev = sigma2;
+        sigma2 = u2;                           // Rayleigh quotient of xi^T xi at unit v
+        if (w2 == 0.0)
+            break;
+        const double wn = std::sqrt(w2);
+        for (int64_t j = 0; j < n; ++j)
+            v[j] = (float)(hw[j] / wn);
+        if (it > 1 && std::fabs(sigma2 - prev) <= tol * sigma2)
+            break;
+    }
+    const double sigma1 = std::sqrt(sigma2);
+    if (f2 > 0.0) {
+        out[0] = std::sqrt(e2 / f2);                                    // ||xi - xi~|| / ||xi||
+        out[1] = std::sqrt(std::max(0.0, 1.0 - sigma2 / f2));            // Eckart-Young floor
+        out[2] = sigma2 > 0.0 ? f2 / sigma2 : 0.0;                       // stable rank
+    }
+    out[3] = sigma1;
+    out[4] = std::sqrt(f2);
+    out[5] = (double)std::min(it, max_iters);
+    return RIKFAD_OK;
 }
 
 }  // extern "C"

@@ -143,6 +143,13 @@ __global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams 
             continue;
         }
         const PanelDev pd = c.panels[pc.panel];
+        if (td.full) {      // element-wise friction: P already holds P_{n+1}
+            if (S != D)
+                for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps)
+                    for (int j = lane; j < pd.width; j += 32)
+                        D[row * td.cols + pd.col0 + j] = S[row * td.cols + pd.col0 + j];
+            continue;
+        }
         const float *C = c.fac + td.fac_off + td.rows + pd.col0;
         for (int j = threadIdx.x; j < pd.width; j += kThreads)
             Cs[j] = C[j];

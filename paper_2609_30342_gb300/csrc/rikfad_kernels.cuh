@@ -340,6 +340,86 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
     }
 }
 
+// ------------------------------ matrix with element-wise friction (full iKFAD)
+//
+// Full iKFAD on a matrix (Eqs. ikfad_1 to ikfad_3, the same expression as
+// vector_element) with the squares of the half-damped momentum P^(1) also
+// summed per row and per column, so the matrix's R, C follow R-iKFAD's factor
+// filter as shadow factors of the same trajectory (the comparison of the
+// paper's Section 4.4).  P holds P_{n+1}.
+__device__ __forceinline__ float full_element(float &x, float &p, float &xi, float g,
+                                              const StepParams &a)
+{
+    const float p_b = fmaf(-a.h, g, p);                       // B
+    x = fmaf(a.h, p_b, x);                                    // A
+    const float p1 = p_b * exp2f(a.ex_cur * xi);              // C, first half-damp
+    xi = fmaf(a.gain, p1 * p1, a.decay * xi);                 // C, friction filter
+    p = (p1 * exp2f(a.ex_cur * xi)) * a.damp_cur;             // C, second half-damp; D
+    return p1 * p1;
+}
+
+template <typename GT>
+__device__ __forceinline__ void matrix_piece_full(const StepParams &a, const PieceDev &pc,
+                                                  const TensorDev &td, const PanelDev &pd,
+                                                  float *red)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t n = td.cols;
+    const int w = pd.width;
+    float *X = a.xptr[pc.tensor];
+    const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
+    float *P = a.pptr[pc.tensor];
+    float *XI = a.fac + td.xi_off;
+    float *rowpart = a.rowpart + td.rowpart_off + (int64_t)(pc.panel - td.panel0) * td.rows;
+    float *myred = red + warp * kPanelMax;
+    for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
+        const int64_t base = row * n + pd.col0;
+        float racc = 0.f;
+        if (td.vec) {
+#pragma unroll 1
+            for (int ch = 0; ch < pd.nch; ++ch) {
+                const int c = ch * kChunk + lane * 8;
+                if (c < w) {
+                    Grad8<GT> gv;
+                    gv.load(G + base + c);
+                    float x[8], p[8], xi[8];
+                    load8(X + base + c, x);
+                    load8(P + base + c, p);
+                    load8(XI + base + c, xi);
+                    float q[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        q[e] = full_element(x[e], p[e], xi[e], gv.get(e), a);
+                        racc += q[e];
+                    }
+                    store8(X + base + c, x);
+                    store8(P + base + c, p);
+                    store8(XI + base + c, xi);
+                    float4 *r4 = reinterpret_cast<float4 *>(myred + c);
+                    float4 r0 = r4[0], r1 = r4[1];
+                    r0.x += q[0]; r0.y += q[1]; r0.z += q[2]; r0.w += q[3];
+                    r1.x += q[4]; r1.y += q[5]; r1.z += q[6]; r1.w += q[7];
+                    r4[0] = r0;
+                    r4[1] = r1;
+                }
+            }
+        } else {
+            for (int c = lane; c < w; c += 32) {
+                float x = X[base + c], p = P[base + c], xi = XI[base + c];
+                const float q = full_element(x, p, xi, grad_at(G, base + c), a);
+                X[base + c] = x;
+                P[base + c] = p;
+                XI[base + c] = xi;
+                racc += q;
+                myred[c] += q;
+            }
+        }
+        racc = warp_sum(racc);
+        if (lane == 0)
+            rowpart[row] = racc;
+    }
+}
+
 // ------------------------------------------------------ the step kernel
 
 // Blocks per SM the register budget is sized for (2: 128 registers/thread).
@@ -347,7 +427,10 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
 #define RIKFAD_STEP_MIN_BLOCKS 2
 #endif
 
-template <typename GT, bool REUSE>
+// SHADOW: the instantiation for handles whose matrices keep element-wise
+// friction with shadow factors (the R-iKFAD instantiation carries no code for
+// it).
+template <typename GT, bool REUSE, bool SHADOW = false>
 __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_kernel(StepParams a)
 {
     __shared__ __align__(16) float Cs[kPanelMax];
@@ -373,7 +456,9 @@ __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_
             red[i] = 0.f;
         const float inv = inv_denominator(row_total(a.spart, td), a.eps);
         __syncthreads();
-        if (td.vec) {
+        if (SHADOW && td.full) {
+            matrix_piece_full<GT>(a, pc, td, pd, red);
+        } else if (td.vec) {
             matrix_piece_vec<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
         } else {
             matrix_piece_scalar<GT, REUSE>(a, pc, td, pd, Cs, red, inv);

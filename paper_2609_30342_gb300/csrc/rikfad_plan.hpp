@@ -41,7 +41,9 @@ struct TensorDev {
     int32_t spart_off;    // partial sums of R, one per kFinThreads rows
     int32_t spart_cnt;
     int32_t vec;          // 1: 8-wide vector loads (cols % 8 == 0)
-    int32_t pad_;
+    int32_t full;         // 1: matrix with element-wise friction (full iKFAD) whose R, C are
+                          //    shadow factors fed by the same momentum (diagnostics)
+    int64_t xi_off;       // full: friction of the m x n elements at fac + xi_off (row-major)
 };
 
 struct PanelDev {

@@ -53,7 +53,7 @@ std::string check_shapes(const rikfad_shape *shapes, int ntensors)
 }
 
 std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes, int max_blocks,
-                       Plan &plan)
+                       Plan &plan, bool full_matrices)
 {
     std::string err = check_shapes(shapes, ntensors);
     if (!err.empty())
@@ -83,6 +83,11 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
         } else {
             td.vec = (td.cols % 8 == 0) ? 1 : 0;
             fac += round_up(td.rows + td.cols, 8);
+            if (full_matrices) {
+                td.full = 1;
+                td.xi_off = fac;
+                fac += round_up(td.rows * td.cols, 8);
+            }
             int64_t np = ceil_div(td.cols, kPanelMax);
             int64_t w = ceil_div(td.cols, np);
             if (td.vec)
@@ -99,7 +104,9 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
                 pd.slot_begin = pd.slot_end = 0;
                 if (td.rows > 0)
                     units.push_back({kMatrixRows, t, (int32_t)p.panels.size(), td.rows,
-                                     pd.width * matrix_elem_bytes(grad_bytes), 1});
+                                     pd.width * (full_matrices ? vector_elem_bytes(grad_bytes)
+                                                               : matrix_elem_bytes(grad_bytes)),
+                                     1});
                 p.panels.push_back(pd);
             }
             td.rowpart_off = rowpart;

@@ -38,8 +38,11 @@ std::string check_shapes(const rikfad_shape *shapes, int ntensors);
 
 // Build the plan for at most max_blocks blocks.  grad_bytes is 2 or 4.
 // Returns "" on success or an error message.
+// full_matrices: every matrix keeps element-wise friction (m x n floats)
+// and its R, C become shadow factors (full iKFAD with R-iKFAD's factors
+// carried alongside).
 std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes, int max_blocks,
-                       Plan &plan);
+                       Plan &plan, bool full_matrices = false);
 
 // Bytes of one step that HBM must move for one element (compulsory traffic):
 // matrix element: read grad + X + P, write X + P; vector element: + friction

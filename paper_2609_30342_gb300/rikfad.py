@@ -50,6 +50,9 @@ SIGNATURES = [
     ("rikfad_create_ikfad", ctypes.c_int, [ctypes.POINTER(Shape), ctypes.c_int,
                                            ctypes.POINTER(HParams), ctypes.c_int,
                                            ctypes.POINTER(_VP)]),
+    ("rikfad_create_ikfad_shadow", ctypes.c_int, [ctypes.POINTER(Shape), ctypes.c_int,
+                                                  ctypes.POINTER(HParams), ctypes.c_int,
+                                                  ctypes.POINTER(_VP)]),
     ("rikfad_destroy", None, [_VP]),
     ("rikfad_step", ctypes.c_int, [_VP, ctypes.c_double, _PP, _PP, _PP, _VP]),
     ("rikfad_materialize", ctypes.c_int, [_VP, _PP, _VP]),
@@ -61,6 +64,9 @@ SIGNATURES = [
     ("rikfad_get_factors", ctypes.c_int, [_VP, ctypes.c_int, _VP, _VP]),
     ("rikfad_set_factors", ctypes.c_int, [_VP, ctypes.c_int, _VP, _VP]),
     ("rikfad_read_denominators", ctypes.c_int, [_VP, _VP, _VP]),
+    ("rikfad_get_friction", ctypes.c_int, [_VP, ctypes.c_int, _VP]),
+    ("rikfad_friction_diagnostics", ctypes.c_int, [_VP, ctypes.c_int, ctypes.c_int, ctypes.c_double,
+                                                   ctypes.POINTER(ctypes.c_double), _VP]),
     ("rikfad_state_image_bytes", ctypes.c_size_t, [_VP]),
     ("rikfad_export_state", ctypes.c_int, [_VP, _VP, _VP]),
     ("rikfad_import_state", ctypes.c_int, [_VP, _VP, _VP]),
@@ -182,19 +188,22 @@ class RIKFAD:
     in the paper (Section 2): ``alpha`` factor decay, ``mu`` friction scale,
     ``gamma`` linear damping, ``eps_stab`` stabiliser.  ``method="ikfad"``
     creates full-friction iKFAD instead (element-wise friction on every
-    tensor, ``rikfad_create_ikfad``).
+    tensor, ``rikfad_create_ikfad``); ``method="ikfad_shadow"`` runs full
+    iKFAD with R-iKFAD's factors carried as shadows (``rikfad_create_ikfad_shadow``,
+    for ``friction_diagnostics``).
     """
 
     def __init__(self, shapes, alpha, mu, gamma=0.0, eps_stab=1e-16, grad_dtype="bf16",
                  method="rikfad"):
-        if method not in ("rikfad", "ikfad"):
-            raise ValueError("method must be 'rikfad' or 'ikfad'")
+        if method not in ("rikfad", "ikfad", "ikfad_shadow"):
+            raise ValueError("method must be 'rikfad', 'ikfad' or 'ikfad_shadow'")
         self.method = method
         self.shapes = [(int(m), int(n)) for m, n in shapes]
         self.grad_dtype = GRAD_BF16 if grad_dtype in ("bf16", GRAD_BF16) else GRAD_F32
         hp = HParams(float(alpha), float(mu), float(gamma), float(eps_stab))
         h = ctypes.c_void_p()
-        create = lib().rikfad_create if method == "rikfad" else lib().rikfad_create_ikfad
+        create = {"rikfad": lib().rikfad_create, "ikfad": lib().rikfad_create_ikfad,
+                  "ikfad_shadow": lib().rikfad_create_ikfad_shadow}[method]
         _check(create(_shapes(self.shapes), len(self.shapes), ctypes.byref(hp), self.grad_dtype,
                       ctypes.byref(h)))
         self._h = h
@@ -267,6 +276,24 @@ class RIKFAD:
             C = np.ascontiguousarray(C, np.float32)
             Cp = C.ctypes.data if C.size else None
         _check(lib().rikfad_set_factors(self.handle, int(t), R.ctypes.data if R.size else None, Cp))
+
+    def get_friction(self, t):
+        """Element-wise friction of tensor t (vector, or matrix of a shadow
+        handle) as float32 numpy of the tensor's shape."""
+        if not 0 <= t < len(self.shapes):
+            raise RikfadError(ERR_ARG, "tensor index %d out of range" % t)
+        m, n = self.shapes[t]
+        out = np.zeros(m if n == 0 else (m, n), np.float32)
+        _check(lib().rikfad_get_friction(self.handle, int(t), out.ctypes.data if out.size else 0))
+        return out
+
+    def friction_diagnostics(self, t, max_iters=200, tol=1e-10, stream=None):
+        """(rel_err, eckart_young_floor, stable_rank, sigma1, frob, iterations)
+        of matrix t of a shadow handle."""
+        out = (ctypes.c_double * 6)()
+        _check(lib().rikfad_friction_diagnostics(self.handle, int(t), int(max_iters), float(tol), out,
+                                                 _stream_ptr(stream)))
+        return tuple(out)
 
     def read_denominators(self, stream=None):
         out = np.zeros(max(len(self.shapes), 1), np.float32)
