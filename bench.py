@@ -437,6 +437,173 @@ def run_ours(args, rank, world, local_rank):
     return line
 
 
+# ------------------------------------------------------------ NEXT-4: dense quadratics
+
+G0_M, G0_N, G0_BATCH, G0_STEPS_PER_CALL, G0_H = 6, 5, 65536, 1000, 0.02
+G0_HP = dict(alpha=1.0, mu=1.0, gamma=0.0, eps_stab=0.1)
+G0_METRIC = ("batched BACD integration of R-iKFAD on dense quadratics (Table tab:g0_slopes "
+             "problem), 6x5 systems, system-steps/s, 1 GB300")
+G0_UNIT = "Gsystem-steps/s"
+# FP32 peak of the SMs: 152 SMs x 128 FP32 lanes x 2 flop per FMA x 2.07 GHz.
+FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def g0_flops(m, n):
+    """Algorithmic flops of one BACD step of one m x n system (an exponential
+    counts as one): A vec(X) 2 d^2; per element the friction R^_i C_j and its
+    scale (2), two damping exponentials and their products (4), kick (2),
+    drift (2), square (1), row and column sums (2); per row the division
+    R_i / (s + eps) and its share of s (2) and the filter (3); per column the
+    filter (3)."""
+    d = m * n
+    return 2 * d * d + 13 * d + 5 * m + 3 * n
+
+
+def g0_oracle_rate(budget_s, steps_hint=2000):
+    """System-steps/s of the float64 C oracle on single 6x5 systems (one thread)."""
+    import oracle
+    from paper_2609_30342_gb300 import workloads as W
+    A, X, P = W.dense_quadratic_instance(G0_M, G0_N, 1)
+    hp = oracle.HParams(**G0_HP)
+    t0 = time.perf_counter()
+    oracle.dense_quadratic_run(A, X.copy(), P.copy(), np.zeros(G0_M), np.zeros(G0_N), G0_H, hp,
+                               steps_hint, [steps_hint])
+    per = (time.perf_counter() - t0) / steps_hint
+    steps = int(max(steps_hint, min(5e7, budget_s / max(per, 1e-9))))
+    t0 = time.perf_counter()
+    oracle.dense_quadratic_run(A, X.copy(), P.copy(), np.zeros(G0_M), np.zeros(G0_N), G0_H, hp, steps,
+                               [steps])
+    sec = time.perf_counter() - t0
+    return steps / sec, steps, sec
+
+
+def run_g0(args, rank, world, local_rank):
+    import torch
+    from paper_2609_30342_gb300 import rikfad
+    from paper_2609_30342_gb300 import workloads as W
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    init_dist(world, "nccl")
+    rikfad.lib()
+    m, n, B, K = G0_M, G0_N, G0_BATCH, G0_STEPS_PER_CALL
+    # 64 seeded instances tiled over the batch (instance generation is host
+    # numpy); each system is integrated independently.
+    A64, X64, P64 = W.dense_quadratic_batch(m, n, range(1000 * rank, 1000 * rank + 64))
+    reps = B // 64
+    A_h = torch.from_numpy(np.tile(A64, (reps, 1, 1))).pin_memory()
+    X_h = torch.from_numpy(np.tile(X64, (reps, 1, 1))).pin_memory()
+    P_h = torch.from_numpy(np.tile(P64, (reps, 1, 1))).pin_memory()
+    R_h = torch.zeros(B, m).pin_memory()
+    C_h = torch.zeros(B, n).pin_memory()
+    A, X, P, R, C = (t.to(dev) for t in (A_h, X_h, P_h, R_h, C_h))
+    rec = torch.tensor([K], dtype=torch.int64, device=dev)
+    E = torch.zeros(1, B, device=dev)
+    hp = G0_HP
+    stream = torch.cuda.current_stream(dev)
+
+    def call(a, x, p, r, c, e, nsteps=K):
+        rikfad.quadratic_run(a, x, p, r, c, G0_H, hp["alpha"], hp["mu"], hp["gamma"], hp["eps_stab"],
+                             nsteps, rec, e, stream=stream)
+
+    for _ in range(args.warmup):
+        call(A, X, P, R, C, E)
+    torch.cuda.synchronize(dev)
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        uuid = None
+    sampler = ClockSampler(uuid)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.25)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        call(A, X, P, R, C, E)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clocks = sampler.stop()
+    ms_total = ev0.elapsed_time(ev1)
+    ms_max = max_over_ranks(ms_total, world, dev)
+    ms_per_call = ms_max / args.steps
+    value = aggregate(B * K, ms_per_call / 1e3, world) / 1e9
+    flops = g0_flops(m, n) * B * K
+    achieved = flops / (ms_total / args.steps / 1e3) / 1e12
+
+    # End to end through the same call with host buffers: every call copies
+    # A, X, P, R, C in from pinned host memory and X, P, R, C and the energy
+    # back out.
+    outs = [torch.empty_like(t).pin_memory() for t in (X_h, P_h, R_h, C_h)]
+    E_h = torch.empty(1, B).pin_memory()
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for d_t, h_t in zip((A, X, P, R, C), (A_h, X_h, P_h, R_h, C_h)):
+            d_t.copy_(h_t, non_blocking=True)
+        call(A, X, P, R, C, E)
+        for h_t, d_t in zip(outs + [E_h], (X, P, R, C, E)):
+            h_t.copy_(d_t, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
+    h2d = sum(t.numel() * 4 for t in (A_h, X_h, P_h, R_h, C_h))
+    d2h = sum(t.numel() * 4 for t in outs) + E_h.numel() * 4
+    e2e = {"value": round(aggregate(B * K, e2e_s / args.steps, world) / 1e9, 4), "unit": G0_UNIT,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # Latency of one step of a single system (what bounds a long run such as
+    # the paper's t = 1e7 table): 2^16 steps of one system, per table size.
+    lat = {}
+    for (mm, nn) in ((2, 2), (4, 3), (6, 5)):
+        a1, x1, p1 = (torch.from_numpy(v).to(dev) for v in W.dense_quadratic_batch(mm, nn, [1]))
+        r1, c1 = torch.zeros(1, mm, device=dev), torch.zeros(1, nn, device=dev)
+        rikfad.quadratic_run(a1, x1, p1, r1, c1, G0_H, 1.0, 1.0, 0.0, 0.1, 1000, stream=stream)
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        rikfad.quadratic_run(a1, x1, p1, r1, c1, G0_H, 1.0, 1.0, 0.0, 0.1, 1 << 16, stream=stream)
+        s1.record(stream)
+        torch.cuda.synchronize(dev)
+        lat["%dx%d" % (mm, nn)] = round(s0.elapsed_time(s1) * 1e6 / (1 << 16), 1)
+
+    if rank != 0:
+        return None
+    line = {
+        "metric": G0_METRIC, "value": round(value, 4), "unit": G0_UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_call, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded): A = B B^T/d + 0.8 I, X(0) ~ N(0, 0.4^2), P(0) ~ N(0, 0.3^2), "
+                "R(0) = C(0) = 0 (the paper's construction)",
+        "config": {"workload": "%d systems of %d x %d, %d BACD steps per call (one bench step = "
+                               "one call)" % (B, m, n, K),
+                   "hyperparameters": dict(hp, h=G0_H),
+                   "l2": "no flush: A alone is %.0f MB > 129 MB L2, read once per launch"
+                         % (A_h.numel() * 4 / 1e6),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 1),
+                     "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": None,
+                     "kernel": "rikfad_quadratic_kernel<8,8>",
+                     "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 flop x 2.07 GHz",
+                     "flops_per_system_step": g0_flops(m, n)},
+        "e2e": e2e,
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+        "single_system_ns_per_step": lat,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        rate, steps, sec = g0_oracle_rate(10.0)
+        line["cpu_baseline"] = {"value": rate / 1e9, "unit": G0_UNIT, "cores": 1, "kind": "oracle",
+                                "sample": "one 6x5 system, %d steps of the float64 C oracle "
+                                          "(%.1f s), single thread" % (steps, sec)}
+    return line
+
+
 # ------------------------------------------------------------ reference arm
 
 def run_reference(args, rank, world):
@@ -444,6 +611,22 @@ def run_reference(args, rank, world):
     same workload, timed per step on the host cores."""
     if rank != 0:
         return None
+    if args.workload == "g0":
+        budget = 150.0 / max(args.steps + args.warmup, 1)
+        rate, steps, sec = g0_oracle_rate(budget)
+        sample = "one 6x5 system, %d steps of the float64 C oracle per bench step, single thread" % steps
+        value = rate / 1e9
+        return {
+            "impl": "reference", "metric": G0_METRIC, "value": value, "unit": G0_UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": G0_BATCH * G0_STEPS_PER_CALL / rate * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+            "config": {"workload": "%d systems of %d x %d, %d BACD steps per call"
+                                   % (G0_BATCH, G0_M, G0_N, G0_STEPS_PER_CALL)},
+            "cpu_baseline": {"value": value, "unit": G0_UNIT, "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": G0_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }
     named, desc, seed = workload(args.workload)
     budget = 150.0 / max(args.steps + args.warmup, 1)
     label, idx = oracle_sample(named, seed, budget_s=budget)
@@ -469,7 +652,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="gpt2s",
-                    help="gpt2s (default), nano, sweep0..sweep3")
+                    help="gpt2s (default), nano, sweep0..sweep3, or g0 (batched BACD on "
+                         "the paper's dense quadratics)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--method", choices=("rikfad", "ikfad", "ikfad_shadow"), default="rikfad",
                     help="rikfad (default), full-friction ikfad, or ikfad with shadow R-iKFAD factors")
@@ -488,6 +672,8 @@ def main():
             raise SystemExit("--gpus %d needs torchrun with %d processes" % (args.gpus, args.gpus))
     if args.impl == "reference":
         line = run_reference(args, rank, world)
+    elif args.workload == "g0":
+        line = run_g0(args, rank, world, local_rank)
     else:
         line = run_ours(args, rank, world, local_rank)
     if line is not None:

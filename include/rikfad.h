@@ -314,6 +314,55 @@ RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols, double ste
                                           int grad_dtype, float *x, const void *grad, float *p,
                                           float *R, float *C, void *stream);
 
+/*
+ * Batched BACD integration of R-iKFAD on small dense quadratics (the test
+ * problem of the paper's numerical validation of the gamma = 0 rates,
+ * Section 3.2 and Table tab:g0_slopes): for every system s of the batch,
+ *   f_s(X) = 1/2 vec(X)^T A_s vec(X),  grad f_s = A_s vec(X) reshaped m x n,
+ * vec(X) row-major (element a = i n + j), and nsteps steps of size h of the
+ * splitting of Appendix A (B, A, C, D in that order, the factors R (m) and
+ * C (n) updated from the half-damped momentum), in float32.  Damping is
+ * carried so that it survives when one step's damping is below float32
+ * resolution of P (late in long gamma = 0 runs): P_k is formed only for the
+ * energies and the output, and 1^T R is filtered alongside R from the total
+ * of [P^(1)]^2 (equal to the sum of R up to rounding).
+ *
+ *   batch         number of systems, 0 <= batch <= 2^24 (0 does nothing)
+ *   m, n          shape of every system: m >= 1, n >= 1, m n <= 32
+ *   A             device, batch x (m n) x (m n) floats, row-major per system
+ *                 (read only; the method needs no symmetry, the energy
+ *                 below is the paper's only for symmetric A)
+ *   X, P          device, batch x (m n) floats: position and the paper's
+ *                 momentum P_k, read and advanced in place to the state
+ *                 after nsteps steps
+ *   R, C          device, batch x m and batch x n floats: the factors, read
+ *                 and advanced in place (start them at zero, as the paper)
+ *   step          h > 0;  hp as for rikfad_create (gamma enters as D)
+ *   nsteps        number of steps, >= 0
+ *   record        device, nrecord int64 step indices, strictly ascending;
+ *                 for every record[r] in [0, nsteps] the energy
+ *                 E = 1/2 vec(X)^T A vec(X) + 1/2 |P|_F^2 of the state after
+ *                 record[r] steps is written to energy[r * batch + s].  Other
+ *                 entries are skipped and their energies left untouched; a
+ *                 list out of order loses the entries after the first descent.
+ *   energy        device, nrecord x batch floats (written)
+ * The call is asynchronous on `stream`.  It runs the steps in launches of S
+ * steps from its start (S = 65536 for batch <= 32768, a smaller power of two
+ * >= 128 for larger batches, so that no launch runs long); every launch
+ * starts from the stored X, P, R, C.  A run split into consecutive calls at
+ * a multiple of S (the second starting from the first's outputs, its record
+ * indices counted from its own start) is therefore bit-identical to one
+ * call; a split elsewhere agrees to float32 rounding.  Errors:
+ * RIKFAD_ERR_ARG for sizes or hyperparameters out of range or a NULL pointer
+ * that is needed, RIKFAD_ERR_ALIGN for a pointer not aligned to its element
+ * type, RIKFAD_ERR_CUDA for a launch failure; messages via rikfad_last_error.
+ */
+RIKFAD_API int rikfad_quadratic_run(int64_t batch, int64_t m, int64_t n, const float *A, float *X,
+                                    float *P, float *R, float *C, double step,
+                                    const rikfad_hparams *hp, int64_t nsteps,
+                                    const int64_t *record, int64_t nrecord, float *energy,
+                                    void *stream);
+
 /* Last error message of the calling thread ("" if none). */
 RIKFAD_API const char *rikfad_last_error(void);
 

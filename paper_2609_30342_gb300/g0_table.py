@@ -1,0 +1,121 @@
+"""Energy-decay slopes of R-iKFAD with gamma = 0 on small dense quadratics,
+integrated on the GPU (the experiment behind Table tab:g0_slopes of Section
+3.2: BACD splitting at h = 0.02, alpha = mu = 1, to t = 1e7, local slopes of
+log E against log t by least squares on successive decades).
+
+Every (m, n, eps_stab) row is one batched ``rikfad_quadratic_run`` call over
+a batch of seeded instances; the rows run on separate CUDA streams at once.
+Slopes are fitted to energies recorded at points spread evenly in log t.
+
+    python -m paper_2609_30342_gb300.g0_table --T 1e7 --seeds 16
+"""
+import argparse
+import json
+import time
+
+import numpy as np
+
+from . import rikfad, workloads
+
+ROWS = ((0.0, 2, 2), (0.0, 4, 3), (0.0, 6, 5), (0.1, 2, 2), (0.1, 4, 3), (0.1, 6, 5))
+
+
+def decades(T, first=1e3):
+    """Lower ends of the decades [lo, 10 lo] inside [first, T]."""
+    out, lo = [], first
+    while lo * 10 <= T * (1 + 1e-12):
+        out.append(lo)
+        lo *= 10
+    return out
+
+
+def decade_slopes(t, E, lows):
+    """Least-squares slope of log E against log t on each [lo, 10 lo].
+    ``E`` is (len(t), batch); returns (len(lows), batch)."""
+    out = np.empty((len(lows), E.shape[1]))
+    for r, lo in enumerate(lows):
+        sel = (t >= lo * (1 - 1e-9)) & (t <= 10 * lo * (1 + 1e-9))
+        u = np.log(t[sel])
+        u = u - u.mean()
+        v = np.log(E[sel].astype(np.float64))
+        out[r] = (u @ (v - v.mean(axis=0))) / (u @ u)
+    return out
+
+
+class Run:
+    """One batched integration enqueued on its own stream."""
+
+    def __init__(self, m, n, eps, seeds, T, h=0.02, alpha=1.0, mu=1.0, gamma=0.0, per_decade=60):
+        import torch
+        self.m, self.n, self.eps, self.h = m, n, eps, h
+        self.seeds = list(seeds)
+        A, X, P = workloads.dense_quadratic_batch(m, n, self.seeds)
+        dev = torch.device("cuda")
+        b = len(self.seeds)
+        self.A = torch.from_numpy(A).to(dev)
+        self.X = torch.from_numpy(X).to(dev)
+        self.P = torch.from_numpy(P).to(dev)
+        self.R = torch.zeros(b, m, device=dev)
+        self.C = torch.zeros(b, n, device=dev)
+        self.k = workloads.log_records(T, h, per_decade)
+        self.rec = torch.from_numpy(self.k).to(dev)
+        self.E = torch.full((len(self.k), b), float("nan"), device=dev)
+        self.nsteps = int(round(T / h))
+        self.stream = torch.cuda.Stream()
+        self.stream.wait_stream(torch.cuda.current_stream())
+        self.args = (alpha, mu, gamma, eps)
+
+    def launch(self):
+        alpha, mu, gamma, eps = self.args
+        rikfad.quadratic_run(self.A, self.X, self.P, self.R, self.C, self.h, alpha, mu, gamma, eps,
+                             self.nsteps, self.rec, self.E, stream=self.stream)
+
+    def energies(self):
+        self.stream.synchronize()
+        return self.k * self.h, self.E.cpu().numpy()
+
+
+def run_table(T=1e7, seeds=range(1, 17), h=0.02, rows=ROWS, per_decade=60):
+    """Slopes for every row of ``rows``: {(eps, m, n): (lows, slopes (decades x seeds))}."""
+    import torch
+    runs = [Run(m, n, eps, seeds, T, h, per_decade=per_decade) for eps, m, n in rows]
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for r in runs:
+        r.launch()
+    out = {}
+    for (eps, m, n), r in zip(rows, runs):
+        t, E = r.energies()
+        lows = decades(T)
+        out[(eps, m, n)] = (lows, decade_slopes(t, E, lows))
+    return out, time.perf_counter() - t0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--T", type=float, default=1e7)
+    ap.add_argument("--h", type=float, default=0.02)
+    ap.add_argument("--seeds", type=int, default=16, help="instances per row (seeds 1..N)")
+    ap.add_argument("--json", action="store_true")
+    a = ap.parse_args()
+    res, secs = run_table(a.T, range(1, a.seeds + 1), a.h)
+    if a.json:
+        print(json.dumps({"T": a.T, "h": a.h, "seconds": secs,
+                          "rows": [{"eps_stab": e, "m": m, "n": n, "decades": lows,
+                                    "seed1": s[:, 0].round(4).tolist(),
+                                    "median": np.median(s, axis=1).round(4).tolist(),
+                                    "min": s.min(axis=1).round(4).tolist(),
+                                    "max": s.max(axis=1).round(4).tolist()}
+                                   for (e, m, n), (lows, s) in res.items()]}))
+        return
+    print("T = %g, h = %g, %d seeds, %.1f s" % (a.T, a.h, a.seeds, secs))
+    for (e, m, n), (lows, s) in res.items():
+        head = "eps=%-4g %dx%d" % (e, m, n)
+        cells = ["[%g,%g] seed1 %+.3f median %+.3f (%+.3f..%+.3f)"
+                 % (lo, 10 * lo, s[r, 0], np.median(s[r]), s[r].min(), s[r].max())
+                 for r, lo in enumerate(lows)]
+        print(head + "\n  " + "\n  ".join(cells))
+
+
+if __name__ == "__main__":
+    main()

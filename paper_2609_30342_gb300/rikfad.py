@@ -81,6 +81,9 @@ SIGNATURES = [
     ("rikfad_step_matrix_noalloc", ctypes.c_int, [ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
                                                   ctypes.c_double, ctypes.POINTER(HParams),
                                                   ctypes.c_int, _VP, _VP, _VP, _VP, _VP, _VP]),
+    ("rikfad_quadratic_run", ctypes.c_int, [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, _VP, _VP,
+                                            _VP, _VP, _VP, ctypes.c_double, ctypes.POINTER(HParams),
+                                            ctypes.c_int64, _VP, ctypes.c_int64, _VP, _VP]),
     ("rikfad_last_error", ctypes.c_char_p, []),
     ("rikfad_abi_version", ctypes.c_int, []),
 ]
@@ -168,6 +171,33 @@ def step_matrix_noalloc(rows, cols, h, pending_step, alpha, mu, gamma, eps_stab,
     _check(lib().rikfad_step_matrix_noalloc(int(rows), int(cols), float(h), float(pending_step),
                                             ctypes.byref(hp), gd, _ptr(x), _ptr(grad), _ptr(p),
                                             _ptr(R), _ptr(C), _stream_ptr(stream)))
+
+
+def quadratic_run(A, X, P, R, C, h, alpha, mu, gamma, eps_stab, nsteps, record=None, energy=None,
+                  stream=None):
+    """Batched BACD integration on dense quadratics (``rikfad_quadratic_run``).
+
+    ``A`` is (batch, m n, m n), ``X`` and ``P`` (batch, m, n), ``R`` (batch, m),
+    ``C`` (batch, n): contiguous float32 CUDA tensors; X, P, R, C are advanced
+    in place.  ``record`` is an int64 CUDA tensor of ascending step indices and
+    ``energy`` a (len(record), batch) float32 CUDA tensor that receives the
+    energies."""
+    batch, m, n = X.shape
+    for t in (A, X, P, R, C) + ((record, energy) if record is not None else ()):
+        if not t.is_contiguous():
+            raise ValueError("quadratic_run needs contiguous tensors")
+    if tuple(A.shape) != (batch, m * n, m * n) or tuple(P.shape) != (batch, m, n) \
+            or tuple(R.shape) != (batch, m) or tuple(C.shape) != (batch, n):
+        raise ValueError("quadratic_run: inconsistent shapes")
+    nrec = 0
+    if record is not None:
+        nrec = record.numel()
+        if energy is None or tuple(energy.shape) != (nrec, batch):
+            raise ValueError("energy must be (len(record), batch)")
+    hp = HParams(float(alpha), float(mu), float(gamma), float(eps_stab))
+    _check(lib().rikfad_quadratic_run(int(batch), int(m), int(n), _ptr(A), _ptr(X), _ptr(P), _ptr(R),
+                                      _ptr(C), float(h), ctypes.byref(hp), int(nsteps), _ptr(record),
+                                      int(nrec), _ptr(energy), _stream_ptr(stream)))
 
 
 class PointerSet:

@@ -147,3 +147,39 @@ def single_matrix_inputs(m, n, seed, steps, x_std=0.02, g_std=0.01):
     X = (rng.standard_normal((m, n), dtype=np.float32) * np.float32(x_std))
     G = [(rng.standard_normal((m, n), dtype=np.float32) * np.float32(g_std)) for _ in range(steps)]
     return X, np.zeros((m, n), np.float32), G
+
+
+def dense_quadratic_instance(m, n, seed):
+    """Test problem of the gamma = 0 rate validation (Section 3.2, numerical
+    set-up appendix): f(X) = 1/2 vec(X)^T A vec(X) with A = B B^T / d + 0.8 I,
+    d = m n, B standard normal; X(0) ~ N(0, 0.4^2) and P(0) ~ N(0, 0.3^2)
+    element-wise (R(0) = C(0) = 0 is the caller's).  float64, from ``seed``;
+    A is made exactly symmetric."""
+    rng = np.random.default_rng(seed)
+    d = m * n
+    B = rng.standard_normal((d, d))
+    A = B @ B.T / d + 0.8 * np.eye(d)
+    A = 0.5 * (A + A.T)
+    X = 0.4 * rng.standard_normal((m, n))
+    P = 0.3 * rng.standard_normal((m, n))
+    return A, X, P
+
+
+def dense_quadratic_batch(m, n, seeds):
+    """float32 (A, X, P) of shapes (b, d, d), (b, m, n), (b, m, n) for the
+    instances of ``seeds`` (see dense_quadratic_instance)."""
+    inst = [dense_quadratic_instance(m, n, s) for s in seeds]
+    A = np.stack([a for a, _, _ in inst]).astype(np.float32)
+    X = np.stack([x for _, x, _ in inst]).astype(np.float32)
+    P = np.stack([p for _, _, p in inst]).astype(np.float32)
+    return A, X, P
+
+
+def log_records(T, h, per_decade=60, t_min=10.0):
+    """Ascending step indices k with t = k h spread evenly in log t over
+    [t_min, T], plus k = 0 and the last step."""
+    n = int(round(T / h))
+    decades = max(np.log10(T / t_min), 0.0)
+    pts = np.logspace(np.log10(t_min), np.log10(T), max(2, int(round(per_decade * decades)) + 1))
+    k = np.unique(np.concatenate([[0], np.round(pts / h).astype(np.int64), [n]]))
+    return k[(k >= 0) & (k <= n)]

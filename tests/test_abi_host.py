@@ -130,3 +130,36 @@ def test_state_bytes_gpt2s_vs_full_friction():
     N, mats, mn, one_d = workloads.count(GPT2S)
     assert (N, mats, mn, one_d) == (124439808, 74, 218705, 121344)
     assert rikfad.state_bytes_for(GPT2S, True) == 4 * (N + mn + one_d) == 499119428
+
+
+def test_quadratic_run_rejects_bad_arguments_before_any_cuda_call():
+    """rikfad_quadratic_run checks sizes, hyperparameters and pointers on the
+    host and returns RIKFAD_ERR_ARG before touching the GPU."""
+    L = rikfad.lib()
+    hp = rikfad.HParams(1.0, 1.0, 0.0, 0.0)
+    bad_hp = rikfad.HParams(1.0, 0.0, 0.0, 0.0)
+    one = ctypes.c_void_p(64)
+    cases = [
+        (1, 6, 6, hp, 10, 0),          # m n = 36 > 32
+        (1, 0, 3, hp, 10, 0),          # m = 0
+        (1, 2, 2, hp, -1, 0),          # nsteps < 0
+        (-1, 2, 2, hp, 10, 0),         # batch < 0
+        (1, 2, 2, bad_hp, 10, 0),      # mu = 0
+        (1, 2, 2, hp, 10, 3),          # record and energy NULL with nrecord > 0
+    ]
+    for batch, m, n, h, nsteps, nrec in cases:
+        rc = L.rikfad_quadratic_run(batch, m, n, one, one, one, one, one, 0.02, ctypes.byref(h), nsteps,
+                                    None, nrec, None, None)
+        assert rc == rikfad.ERR_ARG, (batch, m, n, nsteps, nrec, rc)
+    rc = L.rikfad_quadratic_run(1, 2, 2, None, one, one, one, one, 0.02, ctypes.byref(hp), 10, None, 0,
+                                None, None)
+    assert rc == rikfad.ERR_ARG
+    rc = L.rikfad_quadratic_run(1, 2, 2, one, one, one, one, one, 0.0, ctypes.byref(hp), 10, None, 0,
+                                None, None)
+    assert rc == rikfad.ERR_ARG
+    rc = L.rikfad_quadratic_run(1, 2, 2, ctypes.c_void_p(66), one, one, one, one, 0.02, ctypes.byref(hp),
+                                10, None, 0, None, None)
+    assert rc == rikfad.ERR_ALIGN
+    # batch = 0 is a no-op that succeeds without a device.
+    assert L.rikfad_quadratic_run(0, 2, 2, None, None, None, None, None, 0.02, ctypes.byref(hp), 10,
+                                  None, 0, None, None) == rikfad.OK

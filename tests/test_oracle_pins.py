@@ -31,12 +31,7 @@ def test_fast_pin(pin):
 def _slopes(m, n, eps, seed, T, h=0.02):
     """Local slopes of log E vs log t on [1e3, 1e4] (and [1e4, 1e5] if T >= 1e5)
     for the dense quadratic of the paper's numerical-validation section."""
-    rng = np.random.default_rng(seed)
-    d = m * n
-    B = rng.standard_normal((d, d))
-    A = B @ B.T / d + 0.8 * np.eye(d)
-    X = 0.4 * rng.standard_normal((m, n))
-    P = 0.3 * rng.standard_normal((m, n))
+    A, X, P = workloads.dense_quadratic_instance(m, n, seed)
     nsteps = int(round(T / h))
     rec = np.unique(np.round(np.logspace(2, np.log10(T), 300) / h).astype(np.int64))
     E = oracle.dense_quadratic_run(A, X, P, np.zeros(m), np.zeros(n), h, HParams(1.0, 1.0, 0.0, eps),
