@@ -3,8 +3,9 @@ integrated on the GPU (the experiment behind Table tab:g0_slopes of Section
 3.2: BACD splitting at h = 0.02, alpha = mu = 1, to t = 1e7, local slopes of
 log E against log t by least squares on successive decades).
 
-Every (m, n, eps_stab) row is one batched ``rikfad_quadratic_run`` call over
-a batch of seeded instances; the rows run on separate CUDA streams at once.
+Every (m, n, eps_stab) row integrates a batch of seeded instances with
+``rikfad_quadratic_run`` on its own CUDA stream; the rows are issued as
+interleaved chunks of 2^19 steps, so they run on the GPU at the same time.
 Slopes are fitted to energies recorded at points spread evenly in log t.
 
     python -m paper_2609_30342_gb300.g0_table --T 1e7 --seeds 16
@@ -66,9 +67,40 @@ class Run:
         self.args = (alpha, mu, gamma, eps)
 
     def launch(self):
+        """The whole run as one call."""
         alpha, mu, gamma, eps = self.args
         rikfad.quadratic_run(self.A, self.X, self.P, self.R, self.C, self.h, alpha, mu, gamma, eps,
                              self.nsteps, self.rec, self.E, stream=self.stream)
+
+    def chunks(self, chunk_steps=1 << 19):
+        """The run as consecutive calls of ``chunk_steps`` steps (a multiple of
+        the library's launch length, so the result is bit-identical to one
+        call), each with its own slice of the record list; returns one
+        callable per chunk.  Interleaving the chunks of several runs keeps
+        the GPU's launch queue shared between their streams, so the runs
+        proceed at the same time."""
+        import torch
+        alpha, mu, gamma, eps = self.args
+        out = []
+        k0 = 0
+        while True:
+            k1 = min(k0 + chunk_steps, self.nsteps)
+            last = k1 == self.nsteps
+            sel = np.nonzero((self.k >= k0) & ((self.k <= k1) if last else (self.k < k1)))[0]
+            if sel.size:
+                r0, r1 = int(sel[0]), int(sel[-1]) + 1
+                rec = torch.from_numpy(self.k[r0:r1] - k0).to(self.rec.device)
+                energy = self.E[r0:r1]
+            else:
+                rec, energy = None, None
+
+            def call(k0=k0, k1=k1, rec=rec, energy=energy):
+                rikfad.quadratic_run(self.A, self.X, self.P, self.R, self.C, self.h, alpha, mu, gamma,
+                                     eps, k1 - k0, rec, energy, stream=self.stream)
+            out.append(call)
+            if last:
+                return out
+            k0 = k1
 
     def energies(self):
         self.stream.synchronize()
@@ -79,10 +111,13 @@ def run_table(T=1e7, seeds=range(1, 17), h=0.02, rows=ROWS, per_decade=60):
     """Slopes for every row of ``rows``: {(eps, m, n): (lows, slopes (decades x seeds))}."""
     import torch
     runs = [Run(m, n, eps, seeds, T, h, per_decade=per_decade) for eps, m, n in rows]
+    parts = [r.chunks() for r in runs]
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for r in runs:
-        r.launch()
+    for c in range(max(len(p) for p in parts)):
+        for p in parts:
+            if c < len(p):
+                p[c]()
     out = {}
     for (eps, m, n), r in zip(rows, runs):
         t, E = r.energies()

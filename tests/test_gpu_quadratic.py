@@ -191,6 +191,24 @@ def test_decade_slope_matches_oracle():
         assert abs(got - ref) < 1e-3, (eps, m, n, got, ref)
 
 
+def test_chunked_run_is_bit_identical_to_one_call():
+    """g0_table issues a long run as calls of 2^19 steps (interleaved with
+    other runs); a run cut into calls at multiples of the launch length
+    equals one call bit for bit, energies included."""
+    one = g0_table.Run(4, 3, 0.1, [1, 2, 3], 4000.0, H)     # 200000 steps
+    one.launch()
+    t, E1 = one.energies()
+    two = g0_table.Run(4, 3, 0.1, [1, 2, 3], 4000.0, H)
+    parts = two.chunks(1 << 16)
+    assert len(parts) == 4
+    for c in parts:
+        c()
+    _, E2 = two.energies()
+    assert np.array_equal(E1, E2)
+    for k in ("X", "P", "R", "C"):
+        assert torch.equal(getattr(one, k), getattr(two, k)), k
+
+
 def test_slopes_reproduce_paper_table_to_1e6():
     """Table tab:g0_slopes, first three decades (t to 1e6, 5e7 steps): the
     seed-1 instance of every row lands within 0.04 (2 x 2) or 0.02 of the
