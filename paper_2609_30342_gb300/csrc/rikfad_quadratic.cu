@@ -10,11 +10,12 @@
 // Lane a of a group owns element a = i n + j (row-major vec(X), as the
 // oracle): its X_a, its momentum and row a of A in registers, plus its own
 // copies of R_i, C_j and 1^T R.  The gradient A vec(X) reads X from shared
-// memory with 128-bit broadcast loads.  [P^(1)]^2 is written three times:
-// row-major with rows padded to NB, column-major with columns padded to MB
-// (padding stays zero), and compact; a row sum, a column sum and the total
-// are then a few 128-bit loads each, added in a fixed order, so the lanes of
-// one row (column) hold bit-identical R_i (C_j).  One warp barrier per step
+// memory with 128-bit broadcast loads.  [P^(1)]^2 is written twice:
+// row-major with rows padded to NB and column-major with columns padded to
+// MB (padding stays zero); a row sum and a column sum are then a few 128-bit
+// loads each, added in a fixed order, so the lanes of one row (column) hold
+// bit-identical R_i (C_j).  The total comes from an xor butterfly of
+// shuffles, which also leaves identical bits in every lane.  One warp barrier per step
 // (everything is exchanged together, double buffered); no global memory
 // inside the step loop but the recorded energies.
 
@@ -54,6 +55,12 @@ namespace {
 
 constexpr int kQThreads = 128;                // 4 warps per block
 constexpr int kQWarps = kQThreads / 32;
+// Blocks per SM the registers are sized for (4: up to 128 registers).  A cap of
+// 64 registers (8 blocks) measured slower in latency and in throughput.
+#ifndef RIKFAD_QUAD_MIN_BLOCKS
+#define RIKFAD_QUAD_MIN_BLOCKS 4
+#endif
+constexpr int kQMinBlocks = RIKFAD_QUAD_MIN_BLOCKS;
 constexpr int64_t kQMaxDim = 32;
 
 struct QuadParams {
@@ -134,12 +141,11 @@ __device__ __forceinline__ float sum_run(const float *p)
 }
 
 template <int MB, int NB>
-__global__ void __launch_bounds__(kQThreads) rikfad_quadratic_kernel(QuadParams q)
+__global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kernel(QuadParams q)
 {
     constexpr int L = QShape<MB, NB>::L;
     constexpr int PAD = QShape<MB, NB>::PAD;
     __shared__ __align__(16) float xs[kQWarps][2][32];
-    __shared__ __align__(16) float sa[kQWarps][2][32];          // [P^(1)]^2, compact
     __shared__ __align__(16) float sr[kQWarps][2][64];          // row-major, rows padded to NB
     __shared__ __align__(16) float sc[kQWarps][2][64];          // column-major, columns padded to MB
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -171,7 +177,6 @@ __global__ void __launch_bounds__(kQThreads) rikfad_quadratic_kernel(QuadParams 
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
         xs[warp][u][lane] = 0.f;
-        sa[warp][u][lane] = 0.f;
         sr[warp][u][lane] = 0.f;
         sr[warp][u][lane + 32] = 0.f;
         sc[warp][u][lane] = 0.f;
@@ -232,15 +237,20 @@ __global__ void __launch_bounds__(kQThreads) rikfad_quadratic_kernel(QuadParams 
         z1 = z2;
         xs[warp][cur ^ 1][lane] = x;
         if (elem) {
-            sa[warp][cur][lane] = p1sq;
             sr[warp][cur][pbase + i * NB + j] = p1sq;
             sc[warp][cur][pbase + j * MB + i] = p1sq;
         }
+        // Total of [P^(1)]^2 over the system: an xor butterfly within the
+        // group.  Partners add the same two numbers, so every lane ends with
+        // the same bits.
+        float tot = elem ? p1sq : 0.f;
+#pragma unroll
+        for (int o = L / 2; o > 0; o >>= 1)
+            tot += __shfl_xor_sync(0xffffffffu, tot, o);
         __syncwarp();
-        // Factor filter: row sum, column sum and total, in a fixed order.
+        // Factor filter: row sum and column sum, in a fixed order.
         const float rs = sum_run<NB>(&sr[warp][cur][pbase + i * NB]);
         const float cs = sum_run<MB>(&sc[warp][cur][pbase + j * MB]);
-        const float tot = sum_run<L>(&sa[warp][cur][base]);
         Ri = fmaf(q.gain, rs, q.decay * Ri);
         Cj = fmaf(q.gain, cs, q.decay * Cj);
         S = fmaf(q.gain, tot, q.decay * S);
