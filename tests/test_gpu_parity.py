@@ -243,14 +243,14 @@ def test_gpt2_nano_shaped_full_model():
 def test_gpt2_small_full_size():
     """GPT2-S list (196 tensors, 124.4M parameters), bf16 gradients (seed 3),
     in the launch configuration the benchmark times: the token embedding,
-    the first block and the final LayerNorm exactly against the oracle after
-    2 steps; every tensor checked for the proved invariants (R, C >= 0,
+    the first and the last block and the final LayerNorm exactly against
+    the oracle after 2 steps; every tensor checked for the proved invariants (R, C >= 0,
     sum R = sum C from zero, finite state)."""
     named = workloads.gpt2_small()
     shapes = [s for _, s in named]
     names = [n for n, _ in named]
     pick = [i for i, n in enumerate(names) if n == "wte" or n.startswith("h0.") or
-            n.startswith("ln_f")]
+            n.startswith("h11.") or n.startswith("ln_f")]
     run, ref = _model_parity(shapes, 3, GPT2S_HP, GPT2S_H, 2, tensors=pick)
     _subset_compare(run, ref, pick, 1e-4, 1e-2, "gpt2s step2 ")
     F = run.factors()
