@@ -36,6 +36,7 @@ UNIT = "Gparams/s"
 HP = dict(alpha=0.0579, mu=1.3637e-6, gamma=0.0, eps_stab=1e-16)
 STEP = 0.0918
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0      # GB300 HBM3e, nominal
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "rikfad_step_kernel__gpt2s.md")
 KERNEL_SOURCES = ["paper_2609_30342_gb300/csrc/rikfad_kernels.cuh",
                   "paper_2609_30342_gb300/csrc/rikfad_plan.hpp",
@@ -313,9 +314,20 @@ def run_ours(args, rank, world, local_rank):
     # --vary-h alternates the step size, so every step applies a pending
     # factor of a different h (two exponentials per matrix element).
     hs = (STEP, 0.9 * STEP) if args.vary_h else (STEP, STEP)
+    # --canonical: every step is followed by the materialise pass, so the
+    # stored momentum is always the paper's P_{n+1} (8 more bytes per matrix
+    # element: P read and written once more).
+    p_arr = rikfad.pointer_array(p)
+    if args.canonical:
+        alg_bytes += 8 * (N - one_d)
+
+    def do_step(i, pt):
+        opt.step(hs[i % 2], ptrs=pt, stream=stream)
+        if args.canonical:
+            opt.materialize(p_arr, stream=stream)
 
     for i in range(args.warmup):
-        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
+        do_step(i, ptrs)
     torch.cuda.synchronize(dev)
 
     # ---- device-timed region: inputs resident in HBM (2.24 GB > 129 MB L2)
@@ -332,7 +344,7 @@ def run_ours(args, rank, world, local_rank):
     time.sleep(0.25)      # let the sampler take its first reading
     ev0.record(stream)
     for i in range(args.steps):
-        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
+        do_step(i, ptrs)
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     barrier(world)
@@ -342,7 +354,7 @@ def run_ours(args, rank, world, local_rank):
     # pass is kept out of the headline timing above).
     opt.profile_enable(True)
     for i in range(args.steps):
-        opt.step(hs[i % 2], ptrs=ptrs, stream=stream)
+        do_step(i, ptrs)
     torch.cuda.synchronize(dev)
     clocks = sampler.stop()
     step_ms, fin_ms, nrec = opt.profile_read()
@@ -352,7 +364,8 @@ def run_ours(args, rank, world, local_rank):
     value = aggregate(N, ms_per_step / 1e3, world) / 1e9
     kern_ms = step_ms / max(nrec, 1)
     peak, peak_src = hbm_peak()
-    achieved = alg_bytes / (kern_ms / 1e3) / 1e9
+    kern_bytes = algorithmic_bytes(shapes, 2, args.method)     # the step kernel's own bytes
+    achieved = kern_bytes / (kern_ms / 1e3) / 1e9
     traffic = ncu_traffic() if args.workload == "gpt2s" and args.method == "rikfad" else None
 
     # ---- end to end: every step brings its bf16 gradients in from pinned host
@@ -367,7 +380,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     for i in range(args.steps):
-        opt.step(hs[i % 2], ptrs=ptrs_host, stream=stream)
+        do_step(i, ptrs_host)
         opt.read_denominators(stream)
     torch.cuda.synchronize(dev)
     e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
@@ -413,13 +426,17 @@ def run_ours(args, rank, world, local_rank):
                    "vector_elements": one_d, "grad_dtype": "bf16", "state_dtype": "f32",
                    "hyperparameters": dict(hp, h=STEP), "method": args.method,
                    "step_size": "alternating %g / %g" % hs if args.vary_h else "constant",
+                   "momentum_form": "canonical after every step (3-pass)" if args.canonical
+                                    else "deferred (P^(1) stored)",
                    "l2": "no flush: %.2f GB of inputs per step > 129 MB L2" % (alg_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "hbm_gbs_step": round(alg_bytes / (ms_per_step / 1e3) / 1e9, 1),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic,
                      "kernel": "rikfad_step_kernel", "peak_source": peak_src,
-                     "algorithmic_bytes_per_launch": alg_bytes,
+                     "peak_nominal": NOMINAL_HBM_GBS,
+                     "frac_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
+                     "algorithmic_bytes_per_launch": kern_bytes,
                      "kernel_ms": round(kern_ms, 5),
                      "finalize_kernel_ms": round(fin_ms / max(nrec, 1), 5),
                      "timing": "CUDA events around every launch on the launching stream, "
@@ -661,6 +678,9 @@ def main():
                     help="with --method ikfad_shadow: per-layer friction diagnostics after timing")
     ap.add_argument("--gamma", type=float, default=HP["gamma"],
                     help="linear damping gamma (default 0, R-iKFAD0)")
+    ap.add_argument("--canonical", action="store_true",
+                    help="materialise P after every step (the 3-pass canonical form, 26 B per "
+                         "matrix element)")
     ap.add_argument("--vary-h", action="store_true",
                     help="alternate the step size between h and 0.9 h")
     args = ap.parse_args()

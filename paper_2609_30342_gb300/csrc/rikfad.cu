@@ -372,8 +372,8 @@ int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool 
         c.ex_prev = (float)(-0.5 * h->pending_step * M_LOG2E);
         c.damp_prev = (float)std::exp(-h->hp.gamma * h->pending_step);
         c.eps = (float)h->hp.eps_stab;
-        rikfad_canonical_kernel<<<h->plan.nblocks, kThreads, 0, stream>>>(c);
-        RK_CUDA(cudaGetLastError(), "launch rikfad_canonical_kernel");
+        RK_CUDA(launch_pdl(rikfad_canonical_kernel, h->plan.nblocks, kThreads, stream, c),
+                "launch rikfad_canonical_kernel");
     }
     if (commit)
         h->pending_step = 0.0;

@@ -130,6 +130,8 @@ __global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams 
 {
     __shared__ float Cs[kPanelMax];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    wait_for_predecessor();
+    allow_successor_launch();
     const int q0 = c.block_piece[blockIdx.x], q1 = c.block_piece[blockIdx.x + 1];
     for (int q = q0; q < q1; ++q) {
         const PieceDev pc = c.pieces[q];
@@ -159,8 +161,35 @@ __global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams 
         for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
             const float a_prev = c.ex_prev * (R[row] * inv);
             const int64_t base = row * td.cols + pd.col0;
-            for (int j = lane; j < pd.width; j += 32)
-                D[base + j] = (S[base + j] * exp2f(a_prev * Cs[j])) * c.damp_prev;
+            if (td.vec) {
+                // 16-byte aligned rows and panels: the whole panel row is
+                // loaded first (at most kPanelMax / 128 float4 per lane), so
+                // every load is in flight before the first in-place store.
+                constexpr int kV = kPanelMax / 128;
+                const float4 *s4 = reinterpret_cast<const float4 *>(S + base);
+                float4 *d4 = reinterpret_cast<float4 *>(D + base);
+                const int w4 = pd.width / 4;
+                float4 v[kV];
+#pragma unroll
+                for (int k = 0; k < kV; ++k)
+                    if (lane + 32 * k < w4)
+                        v[k] = __ldcs(s4 + lane + 32 * k);
+#pragma unroll
+                for (int k = 0; k < kV; ++k) {
+                    const int j4 = lane + 32 * k;
+                    if (j4 < w4) {
+                        const int j = 4 * j4;
+                        v[k].x = (v[k].x * exp2f(a_prev * Cs[j])) * c.damp_prev;
+                        v[k].y = (v[k].y * exp2f(a_prev * Cs[j + 1])) * c.damp_prev;
+                        v[k].z = (v[k].z * exp2f(a_prev * Cs[j + 2])) * c.damp_prev;
+                        v[k].w = (v[k].w * exp2f(a_prev * Cs[j + 3])) * c.damp_prev;
+                        __stcs(d4 + j4, v[k]);
+                    }
+                }
+            } else {
+                for (int j = lane; j < pd.width; j += 32)
+                    D[base + j] = (S[base + j] * exp2f(a_prev * Cs[j])) * c.damp_prev;
+            }
         }
         __syncthreads();
     }

@@ -200,6 +200,12 @@ def quadratic_run(A, X, P, R, C, h, alpha, mu, gamma, eps_stab, nsteps, record=N
                                       int(nrec), _ptr(energy), _stream_ptr(stream)))
 
 
+def pointer_array(tensors):
+    """A packed host array of the tensors' device pointers (kept alive by the
+    caller together with the tensors)."""
+    return _ptr_array(tensors)
+
+
 class PointerSet:
     """Pointer arrays for one (x, grad, p) tensor set, packed once."""
 
@@ -269,7 +275,10 @@ class RIKFAD:
                                  _stream_ptr(stream)))
 
     def materialize(self, p, stream=None):
-        _check(lib().rikfad_materialize(self.handle, _ptr_array(p), _stream_ptr(stream)))
+        """Make the stored momenta canonical in place (``rikfad_materialize``);
+        ``p`` is a list of tensors or an array from ``pointer_array``."""
+        arr = p if isinstance(p, ctypes.Array) else _ptr_array(p)
+        _check(lib().rikfad_materialize(self.handle, arr, _stream_ptr(stream)))
 
     def canonical_momentum(self, p, out, stream=None):
         _check(lib().rikfad_canonical_momentum(self.handle, _ptr_array(p), _ptr_array(out),
