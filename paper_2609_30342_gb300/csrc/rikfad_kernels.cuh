@@ -170,38 +170,49 @@ __device__ __forceinline__ float matrix_element(float &x, float p_hat, float g, 
 
 // ACCUM: add each row's squares into the warp's column buffer (several rows
 // per warp); otherwise store them (one row per warp, buffer not cleared).
-template <typename GT, bool REUSE, bool ACCUM = true>
+// HALF (panels of at most kPanelMax / 2 columns): each half-warp takes its own
+// row, 128 columns per chunk, so a panel whose width is not a multiple of 256
+// still loads 256 columns per warp and round trip; half h accumulates its
+// columns at red[warp][h * kPanelMax / 2 + c].
+template <typename GT, bool REUSE, bool ACCUM = true, bool HALF = false>
 __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const PieceDev &pc,
                                                  const TensorDev &td, const PanelDev &pd,
                                                  const float *Cs, float *red, float inv)
 {
+    constexpr int kRowLanes = HALF ? 16 : 32;           // lanes per row
+    constexpr int kRowChunk = kRowLanes * 8;            // columns per chunk of one row
+    constexpr int kRowsPerWarp = HALF ? 2 : 1;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rl = lane & (kRowLanes - 1), half = HALF ? lane >> 4 : 0;
     const int64_t n = td.cols;
     const int w = pd.width;
+    const int nch = HALF ? (w + kRowChunk - 1) / kRowChunk : pd.nch;
     float *X = a.xptr[pc.tensor];
     const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
     float *P = a.pptr[pc.tensor];
     const float *R = a.fac + td.fac_off;
     float *rowpart = a.rowpart + td.rowpart_off + (int64_t)(pc.panel - td.panel0) * td.rows;
-    float *myred = red + warp * kPanelMax;
+    float *myred = red + warp * kPanelMax + half * (kPanelMax / 2);
 
-    for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps) {
-        const float rhat = R[row] * inv;
+    for (int64_t r0 = pc.begin + kRowsPerWarp * warp; r0 < pc.end; r0 += kRowsPerWarp * kWarps) {
+        const int64_t row = r0 + half;
+        const bool live = !HALF || row < pc.end;        // odd piece: the last half-warp idles
+        const float rhat = live ? R[row] * inv : 0.f;
         const float a_cur = a.ex_cur * rhat;
         const float a_prev = REUSE ? a_cur : a.ex_prev * rhat;
         const int64_t base = row * n + pd.col0;
 
-        // RIKFAD_CHUNK_GROUP 256-column chunks at a time: every load of the
-        // group is issued before any arithmetic on it.
+        // RIKFAD_CHUNK_GROUP chunks at a time: every load of the group is
+        // issued before any arithmetic on it.
         float racc = 0.f;
 #pragma unroll 1
-        for (int g0 = 0; g0 < pd.nch; g0 += RIKFAD_CHUNK_GROUP) {
+        for (int g0 = 0; g0 < nch; g0 += RIKFAD_CHUNK_GROUP) {
             float xv[RIKFAD_CHUNK_GROUP][8], pv[RIKFAD_CHUNK_GROUP][8];
             Grad8<GT> gv[RIKFAD_CHUNK_GROUP];
 #pragma unroll
             for (int k = 0; k < RIKFAD_CHUNK_GROUP; ++k) {
-                const int c = (g0 + k) * kChunk + lane * 8;
-                if (c < w) {
+                const int c = (g0 + k) * kRowChunk + rl * 8;
+                if (live && c < w) {
                     gv[k].load(G + base + c);
                     load8(X + base + c, xv[k]);
                     load8(P + base + c, pv[k]);
@@ -209,8 +220,8 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
             }
 #pragma unroll
             for (int k = 0; k < RIKFAD_CHUNK_GROUP; ++k) {
-                const int c = (g0 + k) * kChunk + lane * 8;
-                if (c < w) {
+                const int c = (g0 + k) * kRowChunk + rl * 8;
+                if (live && c < w) {
                     const float4 c0 = *reinterpret_cast<const float4 *>(Cs + c);
                     const float4 c1 = *reinterpret_cast<const float4 *>(Cs + c + 4);
                     const float cv[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
@@ -241,8 +252,14 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
                 }
             }
         }
-        racc = warp_sum(racc);
-        if (lane == 0)
+        if (HALF) {
+#pragma unroll
+            for (int o = 8; o > 0; o >>= 1)
+                racc += __shfl_xor_sync(0xffffffffu, racc, o);
+        } else {
+            racc = warp_sum(racc);
+        }
+        if (live && rl == 0)
             rowpart[row] = racc;
     }
 }
@@ -430,6 +447,10 @@ __device__ __forceinline__ void matrix_piece_full(const StepParams &a, const Pie
 // SHADOW: the instantiation for handles whose matrices keep element-wise
 // friction with shadow factors (the R-iKFAD instantiation carries no code for
 // it).
+// Panels that take two rows per warp (matrix_piece_vec HALF): at most half of
+// kPanelMax wide, and not a whole number of 256-column chunks.
+__device__ __forceinline__ bool half_rows(int w) { return w <= kPanelMax / 2 && w % kChunk != 0; }
+
 template <typename GT, bool REUSE, bool SHADOW = false>
 __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_kernel(StepParams a)
 {
@@ -458,19 +479,25 @@ __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_
         __syncthreads();
         if (SHADOW && td.full) {
             matrix_piece_full<GT>(a, pc, td, pd, red);
+        } else if (td.vec && half_rows(w)) {
+            matrix_piece_vec<GT, REUSE, true, true>(a, pc, td, pd, Cs, red, inv);
         } else if (td.vec) {
             matrix_piece_vec<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
         } else {
             matrix_piece_scalar<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
         }
         __syncthreads();
-        // Column partial sums of this piece, warps added in order.
+        // Column partial sums of this piece, warps (and half-warps) added in order.
         float *out = a.colpart + pc.colpart_off;
+        const bool halves = td.vec && !(SHADOW && td.full) && half_rows(w);
         for (int c = threadIdx.x; c < w; c += kThreads) {
             float s = 0.f;
 #pragma unroll
-            for (int wi = 0; wi < kWarps; ++wi)
+            for (int wi = 0; wi < kWarps; ++wi) {
                 s += red[wi * kPanelMax + c];
+                if (halves)
+                    s += red[wi * kPanelMax + kPanelMax / 2 + c];
+            }
             out[c] = s;
         }
         __syncthreads();
