@@ -9,6 +9,10 @@ interleaved chunks of 2^19 steps, so they run on the GPU at the same time.
 Slopes are fitted to energies recorded at points spread evenly in log t.
 
     python -m paper_2609_30342_gb300.g0_table --T 1e7 --seeds 16
+    python -m paper_2609_30342_gb300.g0_table --prefactors --seeds 16
+
+The second form measures the parameter dependence of the energy prefactors
+(Table tab:g0_prefactors, m = 3, n = 2, t = 1e4).
 """
 import argparse
 import json
@@ -126,13 +130,67 @@ def run_table(T=1e7, seeds=range(1, 17), h=0.02, rows=ROWS, per_decade=60):
     return out, time.perf_counter() - t0
 
 
+PREFACTOR_GRID = {
+    # quantity: (eps values, alpha and mu values), Table tab:g0_prefactors
+    "tE_over_alpha_mu": ((0.0,), (0.5, 1.0, 2.0)),
+    "E_sqrt_t_over_alpha_mu_sqrt_half_eps": ((0.05, 0.2), (0.5, 1.0)),
+}
+
+
+def prefactor_table(T=1e4, m=3, n=2, seeds=range(1, 17), h=0.02):
+    """The parameter dependence of the energy prefactors (Table
+    tab:g0_prefactors): t E/(alpha mu) with eps_stab = 0 over alpha, mu in
+    {1/2, 1, 2}, and E sqrt(t)/(alpha mu sqrt(eps/2)) over alpha, mu in
+    {1/2, 1}, eps in {0.05, 0.2}, at t = T.  Every (alpha, mu, eps) is one
+    batched run over the seeds, all on their own streams at once.  Returns
+    {quantity: (configs, values (configs x seeds))}."""
+    import torch
+    jobs = []
+    for name, (epss, ams) in PREFACTOR_GRID.items():
+        for al in ams:
+            for mu in ams:
+                for ep in epss:
+                    jobs.append((name, al, mu, ep, Run(m, n, ep, seeds, T, h, alpha=al, mu=mu, per_decade=2)))
+    parts = [j[-1].chunks() for j in jobs]
+    torch.cuda.synchronize()
+    for c in range(max(len(p) for p in parts)):
+        for p in parts:
+            if c < len(p):
+                p[c]()
+    out = {}
+    for name, al, mu, ep, run in jobs:
+        _, E = run.energies()
+        e = E[-1].astype(np.float64)            # the last record is t = T
+        q = T * e / (al * mu) if ep == 0.0 else e * np.sqrt(T) / (al * mu * np.sqrt(ep / 2))
+        cfgs, vals = out.setdefault(name, ([], []))
+        cfgs.append((al, mu, ep))
+        vals.append(q)
+    return {k: (c, np.array(v)) for k, (c, v) in out.items()}
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--T", type=float, default=1e7)
     ap.add_argument("--h", type=float, default=0.02)
     ap.add_argument("--seeds", type=int, default=16, help="instances per row (seeds 1..N)")
     ap.add_argument("--json", action="store_true")
+    ap.add_argument("--prefactors", action="store_true",
+                    help="the prefactor table instead (m = 3, n = 2, t = 1e4 unless --T is given)")
     a = ap.parse_args()
+    if a.prefactors:
+        T = a.T if a.T != 1e7 else 1e4
+        res = prefactor_table(T, 3, 2, range(1, a.seeds + 1), a.h)
+        out = {}
+        for name, (cfgs, v) in res.items():
+            mean = v.mean(axis=0)                       # per seed, over the parameter grid
+            spread = v.max(axis=0) / v.min(axis=0)
+            out[name] = {"configs": cfgs, "seed1_mean": round(float(mean[0]), 4),
+                         "seed1_spread": round(float(spread[0]), 4),
+                         "median_mean": round(float(np.median(mean)), 4),
+                         "median_spread": round(float(np.median(spread)), 4),
+                         "spread_range": [round(float(spread.min()), 4), round(float(spread.max()), 4)]}
+        print(json.dumps({"T": T, "h": a.h, "m": 3, "n": 2, "seeds": a.seeds, "prefactors": out}))
+        return
     res, secs = run_table(a.T, range(1, a.seeds + 1), a.h)
     if a.json:
         print(json.dumps({"T": a.T, "h": a.h, "seconds": secs,

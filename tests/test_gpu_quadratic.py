@@ -236,3 +236,21 @@ def test_slopes_independent_of_step_size():
             t, E = run.energies()
             sl.append(g0_table.decade_slopes(t, E, [1e3, 1e4])[:, 0])
         assert np.all(np.abs(sl[0] - sl[1]) < 2e-3), (eps, m, n, sl)
+
+
+def test_prefactor_table_matches_oracle_and_paper():
+    """Table tab:g0_prefactors on the GPU (m = 3, n = 2, t = 1e4, 17 (alpha,
+    mu, eps) settings x 16 instances): the seed-1 values equal the float64
+    oracle's to 1e-3, and over the instances the median spread stays under
+    the paper's bounds (t E/(alpha mu) moves by less than 30% while alpha mu
+    spans 16x; E sqrt(t)/(alpha mu sqrt(eps/2)) by less than 20%)."""
+    res = g0_table.prefactor_table(1e4, 3, 2, range(1, 17), H)
+    A, X, P = workloads.dense_quadratic_batch(3, 2, [1])
+    n = int(round(1e4 / H))
+    for name, (cfgs, v) in res.items():
+        for (al, mu, ep), q in zip(cfgs, v):
+            E, *_ = _oracle(A[0], X[0], P[0], n, [n], HParams(al, mu, 0.0, ep))
+            ref = 1e4 * E[0] / (al * mu) if ep == 0.0 else E[0] * 100.0 / (al * mu * np.sqrt(ep / 2))
+            assert abs(q[0] / ref - 1) < 1e-3, (name, al, mu, ep, q[0], ref)
+        spread = np.median(v.max(axis=0) / v.min(axis=0))
+        assert spread < (1.3 if name == "tE_over_alpha_mu" else 1.2), (name, spread)
