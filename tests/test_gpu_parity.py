@@ -271,3 +271,94 @@ def test_large_matrix_sweep(shape):
     run, ref = _model_parity([shape], 4, GPT2S_HP, GPT2S_H, 2)
     compare_state(run, ref, 1e-4, 1e-2, "%dx%d step2 " % shape)
     run.close()
+
+
+def test_offsets_beyond_2_31_elements():
+    """Maximum sizes: a 65536 x 40960 matrix (2,684,354,560 elements) and a
+    vector of 2^31 + 8 elements, so element offsets pass 2^31 in every
+    kernel (about 60 GB of device memory).  Gradients follow an exact integer
+    pattern (bf16-exact), rebuilt on the host for the sampled rows, columns
+    and elements.
+      Step 1 (zero factors): sampled rows' X and R_i equal the oracle run on
+    that row alone (with no friction yet, a row's update and its R_i depend
+    on the row only), sampled columns' C_j the oracle run on that column
+    alone, and the stored momentum equals the kick -h g exactly (zero
+    friction reduces the step to symplectic Euler); sum R = sum C.
+      Step 2: the vector's sampled elements against the oracle (element-wise
+    rule) for both steps; for the matrix R, C >= 0, sum R = sum C, finite
+    state, and the factor filter R_i <- e^{-alpha h} R_i + k sum_j (P^(1)_ij)^2
+    on sampled rows."""
+    free = torch.cuda.mem_get_info()[0]
+    if free < 75e9:
+        pytest.skip("needs about 60 GB of free device memory")
+    M, N = 65536, 40960
+    V = (1 << 31) + 8
+    hp = HParams(alpha=0.5, mu=1.0, gamma=0.02, eps_stab=1e-8)
+    h = 0.05
+    dev = torch.device("cuda")
+    sc = 2.0 ** -12
+
+    def row_pattern(i, cols):   # host copy of the matrix gradient, float64 (exact)
+        return ((((i * 37) % 255) + (cols * 11) % 255) % 255 - 127) * sc
+
+    a = (torch.arange(M, device=dev, dtype=torch.int32) * 37) % 255
+    b = (torch.arange(N, device=dev, dtype=torch.int32) * 11) % 255
+    G = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
+    for r0 in range(0, M, 4096):
+        blk = (a[r0:r0 + 4096, None] + b[None, :]) % 255 - 127
+        G[r0:r0 + 4096] = (blk.to(torch.float32) * sc).to(torch.bfloat16)
+        del blk
+    gv = torch.empty(V, dtype=torch.bfloat16, device=dev)
+    for e0 in range(0, V, 1 << 27):
+        e = torch.arange(e0, min(V, e0 + (1 << 27)), device=dev, dtype=torch.int64)
+        gv[e0:e0 + e.numel()] = ((((e * 37) % 255) - 127).to(torch.float32) * sc).to(torch.bfloat16)
+        del e
+    X = [torch.zeros(M, N, device=dev), torch.zeros(V, device=dev)]
+    P = [torch.zeros(M, N, device=dev), torch.zeros(V, device=dev)]
+    opt = rikfad.RIKFAD([(M, N), (V, 0)], hp.alpha, hp.mu, hp.gamma, hp.eps_stab, "bf16")
+    ptrs = opt.pack(X, [G, gv], P)
+    opt.step(h, ptrs=ptrs)
+    torch.cuda.synchronize()
+
+    cols = np.arange(N)
+    rows_s = [0, 1, 32767, 52429, M - 1]          # 52429 x 40960 > 2^31
+    cols_s = [0, 1, 20000, N - 1]
+    R1, C1 = opt.get_factors(0)
+    for i in rows_s:
+        g = row_pattern(i, cols)
+        Xo, Po, Ro, Co = np.zeros((1, N)), np.zeros((1, N)), np.zeros(1), np.zeros(N)
+        oracle.step_matrix(Xo, Po, Ro, Co, g[None, :], h, hp)
+        compare("X row %d" % i, X[0][i].double().cpu().numpy(), Xo[0], 1e-5, 1e-2)
+        compare("P^(1) row %d" % i, P[0][i].double().cpu().numpy(), -h * g, 1e-5, 1e-2)
+        assert abs(R1[i] / Ro[0] - 1) < 1e-5, (i, R1[i], Ro[0])
+    for j in cols_s:
+        g = ((((np.arange(M) * 37) % 255) + (j * 11) % 255) % 255 - 127) * sc
+        Xo, Po, Ro, Co = np.zeros((M, 1)), np.zeros((M, 1)), np.zeros(M), np.zeros(1)
+        oracle.step_matrix(Xo, Po, Ro, Co, g[:, None], h, hp)
+        assert abs(C1[j] / Co[0] - 1) < 1e-5, (j, C1[j], Co[0])
+    assert abs(R1.astype(np.float64).sum() / C1.astype(np.float64).sum() - 1) < 1e-5
+
+    opt.step(h, ptrs=ptrs)
+    torch.cuda.synchronize()
+    # Vector: element-wise, so the oracle runs on the sampled elements alone.
+    es = np.array([0, 1, (1 << 31) - 1, 1 << 31, V - 1], dtype=np.int64)
+    ge = (((es * 37) % 255) - 127) * sc
+    xo, po, xio = np.zeros(len(es)), np.zeros(len(es)), np.zeros(len(es))
+    for _ in range(2):
+        oracle.step_vector(xo, po, xio, ge, h, hp)
+    idx = torch.from_numpy(es).to(dev)
+    compare("vector X", X[1][idx].double().cpu().numpy(), xo, 1e-4, 1e-2)
+    compare("vector P", P[1][idx].double().cpu().numpy(), po, 1e-4, 1e-2)
+    # Matrix: invariants and the factor filter on sampled rows.
+    R2, C2 = opt.get_factors(0)
+    assert np.all(R2 >= 0) and np.all(C2 >= 0) and np.all(np.isfinite(R2)) and np.all(np.isfinite(C2))
+    assert abs(R2.astype(np.float64).sum() / C2.astype(np.float64).sum() - 1) < 1e-5
+    d = np.exp(-hp.alpha * h)
+    k = -np.expm1(-hp.alpha * h) / (hp.mu * hp.alpha)
+    for i in rows_s:
+        p1 = P[0][i].double().cpu().numpy()
+        assert np.all(np.isfinite(p1))
+        want = d * R1[i] + k * np.sum(p1 * p1)
+        assert abs(R2[i] / want - 1) < 1e-5, (i, R2[i], want)
+    assert bool(torch.isfinite(X[0]).all()) and bool(torch.isfinite(X[1]).all())
+    opt.close()
