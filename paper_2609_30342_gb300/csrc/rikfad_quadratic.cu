@@ -32,14 +32,17 @@
 // one step's damping h/2 xi~ is ~1e-7: below half a float32 ulp of P, so a
 // stored P (1 - 1e-7) rounds back to P and the damping is lost (the decay
 // slopes bend from -1 to -0.7).  The kernel therefore never stores a damped
-// momentum between steps: it carries P^(B)_{k-1} and the pending exponent
-// z = -h/2 xi~_{k-1}, and forms the next kick as
-//   P^(B)_k = P^(B)_{k-1} + [P^(B)_{k-1} expm1(z - h/2 xi~_k - gamma h) - h g]
+// momentum between steps: it carries P^(B)_{k-1} and the pending
+// e1 = expm1(-h/2 xi~_{k-1}), and forms the next kick as
+//   P^(B)_k = P^(B)_{k-1} + [P^(B)_{k-1} em - h g],
+//   em = expm1(-h/2 xi~_{k-1} - h/2 xi~_k - gamma h)
+//      = (1 + e1)(1 + e2)(1 + expm1(-gamma h)) - 1,  e2 = expm1(-h/2 xi~_k),
 // in which the damping is part of a bracket about 50 times smaller than P,
 // represented to its own float32 precision; the one rounding of the sum is
-// unbiased.  P_k itself (for the energy and the output) is
-// P^(B)_{k-1} + P^(B)_{k-1} expm1(...).  A launch starts from the stored P_k
-// with nothing pending, so runs split at a launch boundary are bit-identical.
+// unbiased.  e2 also gives this step's first half-damp, so one expm1 per
+// step serves both.  P_k itself (for the energy and the output) is
+// P^(B)_{k-1} + P^(B)_{k-1} em.  A launch starts from the stored P_k with
+// nothing pending, so runs split at a launch boundary are bit-identical.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -55,10 +58,10 @@ namespace {
 
 constexpr int kQThreads = 128;                // 4 warps per block
 constexpr int kQWarps = kQThreads / 32;
-// Blocks per SM the registers are sized for (4: up to 128 registers).  A cap of
+// Blocks per SM the registers are sized for (5: up to 102 registers).  A cap of
 // 64 registers (8 blocks) measured slower in latency and in throughput.
 #ifndef RIKFAD_QUAD_MIN_BLOCKS
-#define RIKFAD_QUAD_MIN_BLOCKS 4
+#define RIKFAD_QUAD_MIN_BLOCKS 5
 #endif
 constexpr int kQMinBlocks = RIKFAD_QUAD_MIN_BLOCKS;
 constexpr int64_t kQMaxDim = 32;
@@ -72,7 +75,7 @@ struct QuadParams {
     int64_t nrecord;
     float *energy;
     int64_t k0, k1;                           // this launch runs steps k0 .. k1 - 1 and stops at k1
-    float h, half_h, mgh, decay, gain, eps;   // half_h = -h/2, mgh = -gamma h
+    float h, half_h, eg, decay, gain, eps;    // half_h = -h/2, eg = expm1(-gamma h)
 };
 
 // First index r with record[r] >= k (record ascending).
@@ -172,7 +175,7 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
         for (int t = 0; t < m; ++t)
             S += q.R[sys * m + t];
     }
-    float z1 = 0.f;                           // pending exponent -h/2 xi~_{k-1}
+    float e1 = 0.f;                           // pending expm1(-h/2 xi~_{k-1})
     int cur = 0;
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
@@ -195,7 +198,14 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
         const float den = S + q.eps;
         const float inv = den > 0.f ? __fdividef(1.f, den) : 0.f;
         const float z2 = ((Ri * inv) * Cj) * q.half_h;
-        const float em = s == 0 ? 0.f : expm1_small((z1 + z2) + q.mgh);
+        const float e2 = expm1_small(z2);
+        // expm1 of the owed exponent -h/2 (xi~_{k-1} + xi~_k) - gamma h from
+        // the two half-damps' expm1 values: (1 + e1)(1 + e2)(1 + eg) - 1,
+        // every term of one sign (no cancellation).
+        float em = fmaf(e1, e2, e1 + e2);
+        em = fmaf(q.eg, 1.f + em, em);
+        if (s == 0)
+            em = 0.f;
         // g = A vec(X), four partial sums over groups of four columns.
         const float4 *xv = reinterpret_cast<const float4 *>(&xs[warp][cur][base]);
         float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
@@ -232,9 +242,9 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
         }
         pb = pb + fmaf(-q.h, g, pb * em);     // B (with the owed damping)
         x = fmaf(q.h, pb, x);                 // A
-        const float p1 = fmaf(pb, expm1_small(z2), pb);   // C, first half
+        const float p1 = fmaf(pb, e2, pb);    // C, first half
         const float p1sq = p1 * p1;
-        z1 = z2;
+        e1 = e2;
         xs[warp][cur ^ 1][lane] = x;
         if (elem) {
             sr[warp][cur][pbase + i * NB + j] = p1sq;
@@ -358,7 +368,7 @@ extern "C" RIKFAD_API int rikfad_quadratic_run(int64_t batch, int64_t m, int64_t
     q.energy = energy;
     q.h = (float)step;
     q.half_h = (float)(-0.5 * step);
-    q.mgh = (float)(-hp->gamma * step);
+    q.eg = (float)std::expm1(-hp->gamma * step);
     q.decay = (float)std::exp(-hp->alpha * step);
     q.gain = std::isinf(hp->mu) ? 0.f : (float)(-std::expm1(-hp->alpha * step) / (hp->mu * hp->alpha));
     q.eps = (float)hp->eps_stab;
