@@ -73,6 +73,7 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
             } else {
                 float acc = 0.f;
                 const float *rp = f.rowpart + td.rowpart_off + i;
+#pragma unroll 4
                 for (int k = 0; k < td.npanels; ++k)
                     acc += rp[(int64_t)k * td.rows];
                 val = fmaf(f.gain, acc, f.decay * R[i]);
@@ -90,12 +91,23 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
                 f.spart[td.spart_off + it.chunk] = v;
         }
     } else if (!f.resum_only && it.chunk == 0) {
+        // A panel's slots are consecutive in colpart, pd.width apart (the
+        // planner checks this), so every slot's load is issued at once and
+        // the sum is still taken in slot order.
         const PanelDev pd = f.panels[it.panel];
         const int64_t c = it.begin + threadIdx.x;
         if (c < it.end) {
+            const int ns = pd.slot_end - pd.slot_begin;
+            const float *cp = f.colpart + (ns > 0 ? f.slot_off[pd.slot_begin] : 0) + c;
+            float v[kFinSplitSlots];
+#pragma unroll
+            for (int u = 0; u < kFinSplitSlots; ++u)
+                v[u] = u < ns ? cp[(int64_t)u * pd.width] : 0.f;
             float acc = 0.f;
-            for (int s = pd.slot_begin; s < pd.slot_end; ++s)
-                acc += f.colpart[f.slot_off[s] + c];
+#pragma unroll
+            for (int u = 0; u < kFinSplitSlots; ++u)
+                if (u < ns)
+                    acc += v[u];
             float *C = f.fac + td.fac_off + td.rows + pd.col0;
             C[c] = fmaf(f.gain, acc, f.decay * C[c]);
         }
@@ -104,9 +116,10 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
         const int64_t c = it.begin + lane;
         float acc = 0.f;
         if (c < it.end) {
+            const float *cp = f.colpart + f.slot_off[pd.slot_begin] + c;
 #pragma unroll 4
-            for (int s = pd.slot_begin + warp; s < pd.slot_end; s += kFinThreads / 32)
-                acc += f.colpart[f.slot_off[s] + c];
+            for (int s = warp; s < pd.slot_end - pd.slot_begin; s += kFinThreads / 32)
+                acc += cp[(int64_t)s * pd.width];
         }
         csum[warp][lane] = acc;
         __syncthreads();

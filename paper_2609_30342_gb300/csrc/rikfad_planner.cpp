@@ -183,6 +183,13 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
         p.colpart_floats = colpart;
     }
 
+    // The finalise kernel addresses a panel's slots from its first one: they
+    // must be consecutive and one panel width apart in colpart.
+    for (const PanelDev &pd : p.panels)
+        for (int32_t s = pd.slot_begin; s < pd.slot_end; ++s)
+            if (p.slot_off[s] != p.slot_off[pd.slot_begin] + (int64_t)(s - pd.slot_begin) * pd.width)
+                return "internal: slots of a panel are not contiguous";
+
     // Finalise work: R in chunks of kFinThreads rows (each also yields one
     // partial sum of R), C in chunks of kFinColChunk columns of each panel.
     for (int t = 0; t < ntensors; ++t) {
