@@ -65,6 +65,7 @@ constexpr int kQWarps = kQThreads / 32;
 #endif
 constexpr int kQMinBlocks = RIKFAD_QUAD_MIN_BLOCKS;
 constexpr int64_t kQMaxDim = 32;
+constexpr int kQBufFloats = 128;             // per warp and parity, for each padded copy
 
 struct QuadParams {
     int64_t batch;
@@ -116,8 +117,13 @@ __device__ __forceinline__ float expm1_small(float z)
 template <int MB, int NB>
 struct QShape {
     static constexpr int L = MB * NB >= 32 ? 32 : (MB * NB < 4 ? 4 : MB * NB);   // lanes per system
-    static constexpr int PAD = 2 * L;                  // padded floats per system (>= MB NB)
-    static_assert(MB * NB <= PAD, "padded block must fit");
+    // Row stride of the row-major copy and column stride of the column-major
+    // copy: an extent that is a multiple of 8 floats gets 4 more, so that
+    // consecutive rows (columns) start in different 16-byte bank groups.
+    static constexpr int RS = NB % 8 == 0 ? NB + 4 : NB;
+    static constexpr int CS = MB % 8 == 0 ? MB + 4 : MB;
+    static constexpr int BLK = ((MB * RS > NB * CS ? MB * RS : NB * CS) + 3) / 4 * 4;   // floats per system
+    static_assert((32 / L) * BLK <= kQBufFloats, "padded blocks must fit the warp's buffer");
 };
 
 // Sum of K consecutive floats at p (16-byte aligned when K >= 4), in a fixed order.
@@ -147,14 +153,16 @@ template <int MB, int NB>
 __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kernel(QuadParams q)
 {
     constexpr int L = QShape<MB, NB>::L;
-    constexpr int PAD = QShape<MB, NB>::PAD;
+    constexpr int RS = QShape<MB, NB>::RS;
+    constexpr int CS = QShape<MB, NB>::CS;
+    constexpr int BLK = QShape<MB, NB>::BLK;
     __shared__ __align__(16) float xs[kQWarps][2][32];
-    __shared__ __align__(16) float sr[kQWarps][2][64];          // row-major, rows padded to NB
-    __shared__ __align__(16) float sc[kQWarps][2][64];          // column-major, columns padded to MB
+    __shared__ __align__(16) float sr[kQWarps][2][kQBufFloats];  // row-major, row stride RS
+    __shared__ __align__(16) float sc[kQWarps][2][kQBufFloats];  // column-major, column stride CS
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int a = lane & (L - 1);             // element within the system
     const int base = lane - a;                // first lane of the system's group
-    const int pbase = (lane / L) * PAD;       // the system's padded blocks
+    const int pbase = (lane / L) * BLK;       // the system's padded blocks
     const int64_t sys = ((int64_t)blockIdx.x * kQWarps + warp) * (32 / L) + lane / L;
     const bool live = sys < q.batch;
     const int m = q.m, n = q.n, d = q.d;
@@ -180,10 +188,11 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
         xs[warp][u][lane] = 0.f;
-        sr[warp][u][lane] = 0.f;
-        sr[warp][u][lane + 32] = 0.f;
-        sc[warp][u][lane] = 0.f;
-        sc[warp][u][lane + 32] = 0.f;
+#pragma unroll
+        for (int v = 0; v < kQBufFloats; v += 32) {
+            sr[warp][u][lane + v] = 0.f;
+            sc[warp][u][lane + v] = 0.f;
+        }
     }
     __syncwarp();
     xs[warp][0][lane] = x;
@@ -247,8 +256,8 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
         e1 = e2;
         xs[warp][cur ^ 1][lane] = x;
         if (elem) {
-            sr[warp][cur][pbase + i * NB + j] = p1sq;
-            sc[warp][cur][pbase + j * MB + i] = p1sq;
+            sr[warp][cur][pbase + i * RS + j] = p1sq;
+            sc[warp][cur][pbase + j * CS + i] = p1sq;
         }
         // Total of [P^(1)]^2 over the system: an xor butterfly within the
         // group.  Partners add the same two numbers, so every lane ends with
@@ -259,8 +268,8 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
             tot += __shfl_xor_sync(0xffffffffu, tot, o);
         __syncwarp();
         // Factor filter: row sum and column sum, in a fixed order.
-        const float rs = sum_run<NB>(&sr[warp][cur][pbase + i * NB]);
-        const float cs = sum_run<MB>(&sc[warp][cur][pbase + j * MB]);
+        const float rs = sum_run<NB>(&sr[warp][cur][pbase + i * RS]);
+        const float cs = sum_run<MB>(&sc[warp][cur][pbase + j * CS]);
         Ri = fmaf(q.gain, rs, q.decay * Ri);
         Cj = fmaf(q.gain, cs, q.decay * Cj);
         S = fmaf(q.gain, tot, q.decay * S);
