@@ -46,6 +46,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstdint>
 #include <string>
 
 #include "rikfad.h"
@@ -78,6 +79,34 @@ struct QuadParams {
     int64_t k0, k1;                           // this launch runs steps k0 .. k1 - 1 and stops at k1
     float h, half_h, eg, decay, gain, eps;    // half_h = -h/2, eg = expm1(-gamma h)
 };
+
+// Two float32 lanes in one 64-bit register, and the paired add and FMA on
+// them (PTX add/fma.rn.f32x2: two independent round-to-nearest operations).
+__device__ __forceinline__ uint64_t pack2(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void unpack2(uint64_t v, float &lo, float &hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
 
 // First index r with record[r] >= k (record ascending).
 __device__ __forceinline__ int64_t first_record_at_or_after(const int64_t *record, int64_t nrecord, int64_t k)
@@ -126,20 +155,25 @@ struct QShape {
     static_assert((32 / L) * BLK <= kQBufFloats, "padded blocks must fit the warp's buffer");
 };
 
-// Sum of K consecutive floats at p (16-byte aligned when K >= 4), in a fixed order.
+// Sum of K consecutive floats at p (16-byte aligned when K >= 4), in a fixed
+// order: for K >= 4 the even- and odd-placed elements are summed as the two
+// halves of paired adds (PTX add.rn.f32x2), then the two halves are added.
 template <int K>
 __device__ __forceinline__ float sum_run(const float *p)
 {
     if constexpr (K >= 4) {
-        const float4 *v = reinterpret_cast<const float4 *>(p);
-        float s0 = 0.f, s1 = 0.f;
+        const ulonglong2 *v = reinterpret_cast<const ulonglong2 *>(p);
+        ulonglong2 w = v[0];
+        uint64_t acc = add2(w.x, w.y);
 #pragma unroll
-        for (int q = 0; q < K / 4; ++q) {
-            const float4 w = v[q];
-            s0 += w.x + w.y;
-            s1 += w.z + w.w;
+        for (int q = 1; q < K / 4; ++q) {
+            w = v[q];
+            acc = add2(acc, w.x);
+            acc = add2(acc, w.y);
         }
-        return s0 + s1;
+        float lo, hi;
+        unpack2(acc, lo, hi);
+        return lo + hi;
     } else {
         float s0 = 0.f;
 #pragma unroll
@@ -170,10 +204,14 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
     const int i = elem ? a / n : 0;
     const int j = elem ? a - i * n : 0;
 
-    float arow[L];
+    // Row a of A as packed pairs (A_a,2c, A_a,2c+1) for the paired FMAs below.
+    uint64_t arow2[L / 2];
 #pragma unroll
-    for (int b = 0; b < L; ++b)
-        arow[b] = (elem && b < d) ? q.A[(sys * d + a) * d + b] : 0.f;
+    for (int c = 0; c < L / 2; ++c) {
+        const float lo = (elem && 2 * c < d) ? q.A[(sys * d + a) * d + 2 * c] : 0.f;
+        const float hi = (elem && 2 * c + 1 < d) ? q.A[(sys * d + a) * d + 2 * c + 1] : 0.f;
+        arow2[c] = pack2(lo, hi);
+    }
     float x = elem ? q.X[sys * d + a] : 0.f;
     float pb = elem ? q.P[sys * d + a] : 0.f;   // P_k0 at the launch's first step, then P^(B)
     float Ri = 0.f, Cj = 0.f, S = 0.f;
@@ -215,17 +253,20 @@ __global__ void __launch_bounds__(kQThreads, kQMinBlocks) rikfad_quadratic_kerne
         em = fmaf(q.eg, 1.f + em, em);
         if (s == 0)
             em = 0.f;
-        // g = A vec(X), four partial sums over groups of four columns.
-        const float4 *xv = reinterpret_cast<const float4 *>(&xs[warp][cur][base]);
-        float g0 = 0.f, g1 = 0.f, g2 = 0.f, g3 = 0.f;
+        // g = A vec(X): four partial sums over the columns 4c, 4c+1, 4c+2,
+        // 4c+3, carried as two pairs and advanced by paired FMAs (each half
+        // a round-to-nearest FMA, so the same arithmetic as four fmaf).
+        const ulonglong2 *xv = reinterpret_cast<const ulonglong2 *>(&xs[warp][cur][base]);
+        uint64_t g01 = 0ull, g23 = 0ull;
 #pragma unroll
         for (int b4 = 0; b4 < L / 4; ++b4) {
-            const float4 v = xv[b4];
-            g0 = fmaf(arow[4 * b4 + 0], v.x, g0);
-            g1 = fmaf(arow[4 * b4 + 1], v.y, g1);
-            g2 = fmaf(arow[4 * b4 + 2], v.z, g2);
-            g3 = fmaf(arow[4 * b4 + 3], v.w, g3);
+            const ulonglong2 v = xv[b4];
+            g01 = fma2(arow2[2 * b4], v.x, g01);
+            g23 = fma2(arow2[2 * b4 + 1], v.y, g23);
         }
+        float g0, g1, g2, g3;
+        unpack2(g01, g0, g1);
+        unpack2(g23, g2, g3);
         const float g = (g0 + g1) + (g2 + g3);
         while (s == next) {                   // energy of the state after k0 + s steps
             const float pk = fmaf(pb, em, pb);
