@@ -23,7 +23,8 @@ import oracle
 from paper_2609_30342_gb300 import rikfad, workloads
 
 
-def compare(name, gpu, ref, rtol, floor):
+def compare(name, gpu, ref, rtol, floor, atol=0.0):
+    """Element-wise |gpu - ref| <= rtol (|ref| + floor rms(ref)) + atol."""
     gpu = np.asarray(gpu, np.float64).ravel()
     ref = np.asarray(ref, np.float64).ravel()
     assert gpu.shape == ref.shape, name
@@ -32,7 +33,7 @@ def compare(name, gpu, ref, rtol, floor):
     assert np.all(np.isfinite(gpu)), "%s: non-finite values" % name
     rms = float(np.sqrt(np.mean(ref * ref)))
     err = np.abs(gpu - ref)
-    bound = rtol * (np.abs(ref) + floor * rms)
+    bound = rtol * (np.abs(ref) + floor * rms) + atol
     bad = err > bound
     with np.errstate(divide="ignore", invalid="ignore"):
         rel = np.where(ref != 0, err / np.abs(ref), np.where(err == 0, 0.0, np.inf))
@@ -101,18 +102,18 @@ def oracle_from_gpu(run):
     return st
 
 
-def compare_state(run, st, rtol, floor, tag="", tensors=None):
+def compare_state(run, st, rtol, floor, tag="", tensors=None, atol=0.0):
     """Compare GPU X, canonical P and factors with the oracle state."""
     Xg, Pg, F = run.X(), run.canonical_P(), run.factors()
     stats = {}
     idx = range(len(run.shapes)) if tensors is None else tensors
     for t in idx:
         n = run.shapes[t][1]
-        stats[("X", t)] = compare("%sX[%d]" % (tag, t), Xg[t], st.X[t], rtol, floor)
-        stats[("P", t)] = compare("%sP[%d]" % (tag, t), Pg[t], st.P[t], rtol, floor)
+        stats[("X", t)] = compare("%sX[%d]" % (tag, t), Xg[t], st.X[t], rtol, floor, atol)
+        stats[("P", t)] = compare("%sP[%d]" % (tag, t), Pg[t], st.P[t], rtol, floor, atol)
         if n == 0:
-            stats[("xi", t)] = compare("%sxi[%d]" % (tag, t), F[t][0], st.xi[t], rtol, floor)
+            stats[("xi", t)] = compare("%sxi[%d]" % (tag, t), F[t][0], st.xi[t], rtol, floor, atol)
         else:
-            stats[("R", t)] = compare("%sR[%d]" % (tag, t), F[t][0], st.R[t], rtol, floor)
-            stats[("C", t)] = compare("%sC[%d]" % (tag, t), F[t][1], st.C[t], rtol, floor)
+            stats[("R", t)] = compare("%sR[%d]" % (tag, t), F[t][0], st.R[t], rtol, floor, atol)
+            stats[("C", t)] = compare("%sC[%d]" % (tag, t), F[t][1], st.C[t], rtol, floor, atol)
     return stats

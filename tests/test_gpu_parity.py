@@ -190,6 +190,45 @@ def test_edge_shapes(grad_bf16, eps, gamma):
     run.close()
 
 
+DEGENERATE = {
+    # mu = inf: the factor filter's gain is zero, so friction never appears
+    # and the step is damped symplectic Euler.
+    "mu_inf": (HParams(alpha=0.3, mu=float("inf"), gamma=0.05, eps_stab=1e-8), 0.05, 1.0),
+    # friction so large that exp(-h/2 xi~) underflows: the momentum is wiped
+    "huge_friction": (HParams(alpha=0.3, mu=1e-12, gamma=0.0, eps_stab=1e-16), 0.05, 10.0),
+    # alpha h = 10: the factors forget everything but the last step
+    "fast_decay": (HParams(alpha=100.0, mu=1e-3, gamma=0.0, eps_stab=1e-8), 0.1, 1.0),
+    # eps_stab far above 1^T R: friction tiny and set by eps
+    "large_eps": (HParams(alpha=0.3, mu=1e-3, gamma=0.0, eps_stab=1e3), 0.05, 1.0),
+    # a tiny step
+    "tiny_h": (HParams(alpha=0.3, mu=1e-3, gamma=0.1, eps_stab=1e-8), 1e-6, 1.0),
+}
+
+
+@pytest.mark.parametrize("case", sorted(DEGENERATE))
+def test_degenerate_hyperparameters(case):
+    """Limits of the method on the edge-shape list (bf16 gradients, 3
+    steps from zero factors): every tensor against the oracle.  Values the
+    oracle keeps below float32's smallest normal number (1.18e-38, reached
+    where exp(-h/2 xi~) underflows) are zero or subnormal in the kernel's
+    float32 state, hence the absolute floor of 1.2e-38."""
+    hp, h, gscale = DEGENERATE[case]
+    rng = np.random.default_rng(11)
+    shapes = EDGE_SHAPES
+    X = [rng.standard_normal(workloads.array_shape(s)).astype(np.float32) for s in shapes]
+    P = [(0.1 * rng.standard_normal(workloads.array_shape(s))).astype(np.float32) for s in shapes]
+    run = GpuRun(shapes, hp, True, X, P)
+    ref = oracle_from_gpu(run)
+    for k in range(3):
+        g = [workloads.bf16_round(gscale * rng.standard_normal(workloads.array_shape(s)).astype(np.float32))
+             for s in shapes]
+        run.set_grads(g)
+        run.step(h)
+        ref.step([a.astype(np.float64) for a in g], h, hp)
+        compare_state(run, ref, 1e-4, 1e-2, "%s step%d " % (case, k + 1), atol=1.2e-38)
+    run.close()
+
+
 # ------------------------------------------------------------ model-sized
 
 def _model_parity(shapes, seed, hp, h, steps, tensors=None):
