@@ -279,6 +279,27 @@ def test_gpt2_nano_shaped_full_model():
     run.close()
 
 
+def test_gpt2_nano_100_steps():
+    """The stated bound after 100 steps on a model-shaped list: the whole
+    GPT2-Nano-shaped list (100 tensors, 30.06M parameters, bf16 gradients,
+    seed 2, the paper's GPT2-S hyperparameters) takes 100 steps on the GPU;
+    the oracle follows the position embedding, the first block and the
+    final LayerNorm (every tensor's update depends only on its own state
+    and gradient), compared at rtol 1e-4 with a floor of 0.1 rms.  Where
+    P_n and h g (or X_n and h P^(B)) nearly cancel, each float32 step
+    leaves an absolute error of about one ulp of an rms-sized term (6e-8
+    rms); over 100 steps that accumulates to ~6e-6 rms, which the floor
+    (1e-5 rms at rtol 1e-4) admits and the one-step floor (1e-6 rms) does
+    not."""
+    named = workloads.gpt2_nano()
+    shapes = [s for _, s in named]
+    names = [n for n, _ in named]
+    pick = [i for i, n in enumerate(names) if n == "wpe" or n.startswith("h0.") or n.startswith("ln_f")]
+    run, ref = _model_parity(shapes, 2, GPT2S_HP, GPT2S_H, 100, tensors=pick)
+    _subset_compare(run, ref, pick, 1e-4, 0.1, "nano step100 ")
+    run.close()
+
+
 def test_gpt2_small_full_size():
     """GPT2-S list (196 tensors, 124.4M parameters), bf16 gradients (seed 3),
     in the launch configuration the benchmark times: the token embedding,
