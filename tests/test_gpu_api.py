@@ -9,7 +9,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import rikfad, workloads
 
-from gpu_helpers import GpuRun, compare, compare_state, oracle_from_gpu
+from gpu_helpers import GpuRun, compare_state
 
 pytestmark = pytest.mark.gpu
 

@@ -3,7 +3,6 @@ GPU (rikfad_create_ikfad_shadow, rikfad_friction_diagnostics) against the
 oracle of the paper's Section 4.4 comparison."""
 import numpy as np
 import pytest
-import torch
 
 from oracle import HParams
 from oracle.diagnostics import friction_metrics, shadow_step

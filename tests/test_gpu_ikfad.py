@@ -2,7 +2,6 @@
 oracle's element-wise rule, and the rank-1 cross-check against R-iKFAD."""
 import numpy as np
 import pytest
-import torch
 
 import oracle
 from oracle import HParams

@@ -7,7 +7,6 @@ mutant that passes every pin would mean the pins cannot see that mistake.
 """
 import os
 import subprocess
-import tempfile
 
 import pytest
 
