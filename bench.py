@@ -52,6 +52,12 @@ def workload(name):
         desc = ("GPT2-S parameter set: 12 layers, width 768, vocab 50257 (tied), ctx 1024, "
                 "separate q/k/v; 74 matrices + 122 vectors")
         seed = 3
+    elif name in ("gpt2m", "gpt2xl"):
+        layers, width = (24, 1024) if name == "gpt2m" else (48, 1600)
+        named = W.gpt2_shapes(layers, width, 50257, 1024)
+        desc = ("GPT2-%s-shaped parameter set: %d layers, width %d, vocab 50257 (tied), ctx 1024, "
+                "separate q/k/v" % ("M" if name == "gpt2m" else "XL", layers, width))
+        seed = 5
     elif name == "nano":
         named = W.gpt2_nano()
         desc = "GPT2-Nano-shaped parameter set: 6 layers, width 384, vocab 50304, ctx 256"
@@ -669,8 +675,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="gpt2s",
-                    help="gpt2s (default), nano, sweep0..sweep3, or g0 (batched BACD on "
-                         "the paper's dense quadratics)")
+                    help="gpt2s (default), nano, gpt2m, gpt2xl, sweep0..sweep3, or g0 (batched "
+                         "BACD on the paper's dense quadratics)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--method", choices=("rikfad", "ikfad", "ikfad_shadow"), default="rikfad",
                     help="rikfad (default), full-friction ikfad, or ikfad with shadow R-iKFAD factors")

@@ -88,10 +88,15 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
                 td.xi_off = fac;
                 fac += round_up(td.rows * td.cols, 8);
             }
+            // Panels of at most kPanelMax columns.  On the 8-wide path a warp
+            // moves one 256-column chunk per round trip, so every panel but
+            // the last is a whole number of chunks: the matrix then takes the
+            // fewest chunks, ceil(cols / 256) per row (two 800-wide panels of
+            // a 1600-wide matrix would take 8, 1024 + 576 take 7).
             int64_t np = ceil_div(td.cols, kPanelMax);
             int64_t w = ceil_div(td.cols, np);
             if (td.vec)
-                w = round_up(w, 8);
+                w = std::min<int64_t>(kPanelMax, round_up(w, kChunk));
             np = ceil_div(td.cols, w);
             td.npanels = (int32_t)np;
             td.panel0 = (int32_t)p.panels.size();
