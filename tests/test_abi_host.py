@@ -163,3 +163,16 @@ def test_quadratic_run_rejects_bad_arguments_before_any_cuda_call():
     # batch = 0 is a no-op that succeeds without a device.
     assert L.rikfad_quadratic_run(0, 2, 2, None, None, None, None, None, 0.02, ctypes.byref(hp), 10,
                                   None, 0, None, None) == rikfad.OK
+
+
+@pytest.mark.parametrize("cols", [8, 40, 384, 576, 768, 800, 1032, 1536, 1600, 2048, 3000, 3072, 6400, 14336])
+def test_panels_are_whole_chunks(cols):
+    """On the 8-wide path (cols a multiple of 8) every column panel of a
+    matrix but its last is a whole number of 256-column chunks and at most
+    1024 wide, so a row takes the fewest chunk round trips, ceil(cols/256)."""
+    plan = rikfad.plan_query([(64, cols)], "bf16", 4)
+    panels = sorted({(int(c0), int(w)) for c0, w in zip(plan[:, 3], plan[:, 4])})
+    assert sum(w for _, w in panels) == cols
+    assert all(w <= 1024 for _, w in panels)
+    assert all(w % 256 == 0 for _, w in panels[:-1]), panels
+    assert sum(-(-w // 256) for _, w in panels) == -(-cols // 256)
