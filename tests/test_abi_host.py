@@ -176,3 +176,41 @@ def test_panels_are_whole_chunks(cols):
     assert all(w <= 1024 for _, w in panels)
     assert all(w % 256 == 0 for _, w in panels[:-1]), panels
     assert sum(-(-w // 256) for _, w in panels) == -(-cols // 256)
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include "rikfad.h"
+int main(void)
+{
+    rikfad_shape shapes[2] = {{768, 768}, {768, 0}};
+    rikfad_hparams bad = {1.0, 0.0, 0.0, 0.0};
+    size_t bytes = rikfad_state_bytes_for(shapes, 2, 1);
+    int64_t rows = rikfad_plan_query(shapes, 2, RIKFAD_GRAD_BF16, 4, NULL, 0);
+    int rc = rikfad_quadratic_run(1, 2, 2, NULL, NULL, NULL, NULL, NULL, 0.02, &bad, 10, NULL, 0,
+                                  NULL, NULL);
+    printf("%d %zu %lld %d\n", rikfad_abi_version(), bytes, (long long)rows, rc);
+    return 0;
+}
+"""
+
+
+def test_plain_c_client(tmp_path):
+    """The boundary is a C ABI: include/rikfad.h compiles as strict C99 and a C
+    program links against the library and calls it (host-only calls)."""
+    import shutil
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(rikfad.LIB_PATH)
+    subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I",
+                    os.path.join(ROOT, "include"), str(src), "-L", libdir, "-lrikfad",
+                    "-Wl,-rpath," + libdir, "-o", str(exe)], check=True, capture_output=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()
+    assert int(out[0]) == rikfad.lib().rikfad_abi_version()
+    assert int(out[1]) == 4 * (768 * 768 + 768 + 768 + 2 * 768)
+    assert int(out[2]) > 0
+    assert int(out[3]) == rikfad.ERR_ARG
