@@ -170,33 +170,34 @@ __device__ __forceinline__ float matrix_element(float &x, float p_hat, float g, 
 
 // ACCUM: add each row's squares into the warp's column buffer (several rows
 // per warp); otherwise store them (one row per warp, buffer not cleared).
-// HALF (panels of at most kPanelMax / 2 columns): each half-warp takes its own
-// row, 128 columns per chunk, so a panel whose width is not a multiple of 256
-// still loads 256 columns per warp and round trip; half h accumulates its
-// columns at red[warp][h * kPanelMax / 2 + c].
-template <typename GT, bool REUSE, bool ACCUM = true, bool HALF = false>
+// RPW rows per warp (1, 2 or 4; panels of at most kPanelMax / RPW columns):
+// each of the warp's RPW lane groups takes its own row, 256 / RPW columns per
+// chunk, so a panel whose width is not a multiple of 256 still loads 256
+// columns per warp and round trip; group h accumulates its columns at
+// red[warp][h * kPanelMax / RPW + c].
+template <typename GT, bool REUSE, bool ACCUM = true, int RPW = 1>
 __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const PieceDev &pc,
                                                  const TensorDev &td, const PanelDev &pd,
                                                  const float *Cs, float *red, float inv)
 {
-    constexpr int kRowLanes = HALF ? 16 : 32;           // lanes per row
+    constexpr int kRowLanes = 32 / RPW;                 // lanes per row
     constexpr int kRowChunk = kRowLanes * 8;            // columns per chunk of one row
-    constexpr int kRowsPerWarp = HALF ? 2 : 1;
+    constexpr int kRowsPerWarp = RPW;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int rl = lane & (kRowLanes - 1), half = HALF ? lane >> 4 : 0;
+    const int rl = lane & (kRowLanes - 1), half = lane / kRowLanes;   // lane group = row
     const int64_t n = td.cols;
     const int w = pd.width;
-    const int nch = HALF ? (w + kRowChunk - 1) / kRowChunk : pd.nch;
+    const int nch = RPW > 1 ? (w + kRowChunk - 1) / kRowChunk : pd.nch;
     float *X = a.xptr[pc.tensor];
     const GT *G = static_cast<const GT *>(a.gptr[pc.tensor]);
     float *P = a.pptr[pc.tensor];
     const float *R = a.fac + td.fac_off;
     float *rowpart = a.rowpart + td.rowpart_off + (int64_t)(pc.panel - td.panel0) * td.rows;
-    float *myred = red + warp * kPanelMax + half * (kPanelMax / 2);
+    float *myred = red + warp * kPanelMax + half * (kPanelMax / RPW);
 
     for (int64_t r0 = pc.begin + kRowsPerWarp * warp; r0 < pc.end; r0 += kRowsPerWarp * kWarps) {
         const int64_t row = r0 + half;
-        const bool live = !HALF || row < pc.end;        // odd piece: the last half-warp idles
+        const bool live = RPW == 1 || row < pc.end;     // ragged piece: trailing lane groups idle
         const float rhat = live ? R[row] * inv : 0.f;
         const float a_cur = a.ex_cur * rhat;
         const float a_prev = REUSE ? a_cur : a.ex_prev * rhat;
@@ -252,9 +253,9 @@ __device__ __forceinline__ void matrix_piece_vec(const StepParams &a, const Piec
                 }
             }
         }
-        if (HALF) {
+        if (RPW > 1) {
 #pragma unroll
-            for (int o = 8; o > 0; o >>= 1)
+            for (int o = kRowLanes / 2; o > 0; o >>= 1)
                 racc += __shfl_xor_sync(0xffffffffu, racc, o);
         } else {
             racc = warp_sum(racc);
@@ -447,9 +448,32 @@ __device__ __forceinline__ void matrix_piece_full(const StepParams &a, const Pie
 // SHADOW: the instantiation for handles whose matrices keep element-wise
 // friction with shadow factors (the R-iKFAD instantiation carries no code for
 // it).
-// Panels that take two rows per warp (matrix_piece_vec HALF): at most half of
-// kPanelMax wide, and not a whole number of 256-column chunks.
-__device__ __forceinline__ bool half_rows(int w) { return w <= kPanelMax / 2 && w % kChunk != 0; }
+// out[c] = the piece's column sums: warp wi's lane group h holds its share at
+// red[wi * kPanelMax + h * kPanelMax / RPW + c]; added warp by warp, groups in
+// order.
+template <int RPW>
+__device__ __forceinline__ void column_partials(const float *red, float *out, int w)
+{
+    for (int c = threadIdx.x; c < w; c += kThreads) {
+        float s = 0.f;
+#pragma unroll
+        for (int wi = 0; wi < kWarps; ++wi)
+#pragma unroll
+            for (int h = 0; h < RPW; ++h)
+                s += red[wi * kPanelMax + h * (kPanelMax / RPW) + c];
+        out[c] = s;
+    }
+}
+
+// Rows per warp for an 8-wide panel (matrix_piece_vec RPW): a panel that is
+// not a whole number of 256-column chunks takes 4 rows per warp up to 64
+// columns and 2 up to kPanelMax / 2 columns; every other panel takes 1.
+__device__ __forceinline__ int rows_per_warp(int w)
+{
+    if (w % kChunk == 0 || w > kPanelMax / 2)
+        return 1;
+    return w <= kChunk / 4 ? 4 : 2;
+}
 
 template <typename GT, bool REUSE, bool SHADOW = false>
 __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_kernel(StepParams a)
@@ -479,27 +503,25 @@ __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_
         __syncthreads();
         if (SHADOW && td.full) {
             matrix_piece_full<GT>(a, pc, td, pd, red);
-        } else if (td.vec && half_rows(w)) {
-            matrix_piece_vec<GT, REUSE, true, true>(a, pc, td, pd, Cs, red, inv);
+        } else if (td.vec && rows_per_warp(w) == 4) {
+            matrix_piece_vec<GT, REUSE, true, 4>(a, pc, td, pd, Cs, red, inv);
+        } else if (td.vec && rows_per_warp(w) == 2) {
+            matrix_piece_vec<GT, REUSE, true, 2>(a, pc, td, pd, Cs, red, inv);
         } else if (td.vec) {
             matrix_piece_vec<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
         } else {
             matrix_piece_scalar<GT, REUSE>(a, pc, td, pd, Cs, red, inv);
         }
         __syncthreads();
-        // Column partial sums of this piece, warps (and half-warps) added in order.
+        // Column partial sums of this piece, warps (and their lane groups) added in order.
         float *out = a.colpart + pc.colpart_off;
-        const bool halves = td.vec && !(SHADOW && td.full) && half_rows(w);
-        for (int c = threadIdx.x; c < w; c += kThreads) {
-            float s = 0.f;
-#pragma unroll
-            for (int wi = 0; wi < kWarps; ++wi) {
-                s += red[wi * kPanelMax + c];
-                if (halves)
-                    s += red[wi * kPanelMax + kPanelMax / 2 + c];
-            }
-            out[c] = s;
-        }
+        const int rpw = td.vec && !(SHADOW && td.full) ? rows_per_warp(w) : 1;
+        if (rpw == 1)
+            column_partials<1>(red, out, w);
+        else if (rpw == 2)
+            column_partials<2>(red, out, w);
+        else
+            column_partials<4>(red, out, w);
         __syncthreads();
     }
 }

@@ -98,13 +98,31 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
             if (td.vec)
                 w = std::min<int64_t>(kPanelMax, round_up(w, kChunk));
             np = ceil_div(td.cols, w);
+            std::vector<int64_t> widths;
+            for (int64_t k = 0; k < np; ++k)
+                widths.push_back(std::min<int64_t>(w, td.cols - k * w));
+            // A last panel wider than kPanelMax / 2 whose tail past whole
+            // chunks is at most half a chunk gives that tail a panel of its
+            // own, which the kernel runs with several rows per warp (1600 =
+            // 1024 + 512 + 64 takes 6.25 round trips per row, 1024 + 576
+            // takes 7).
+            if (td.vec) {
+                const int64_t r = widths.back(), tail = r % kChunk;
+                if (r > kPanelMax / 2 && tail > 0 && tail <= kChunk / 2) {
+                    widths.back() = r - tail;
+                    widths.push_back(tail);
+                }
+            }
+            np = (int64_t)widths.size();
             td.npanels = (int32_t)np;
             td.panel0 = (int32_t)p.panels.size();
+            int64_t col0 = 0;
             for (int64_t k = 0; k < np; ++k) {
                 PanelDev pd{};
                 pd.tensor = t;
-                pd.col0 = (int32_t)(k * w);
-                pd.width = (int32_t)std::min<int64_t>(w, td.cols - k * w);
+                pd.col0 = (int32_t)col0;
+                pd.width = (int32_t)widths[k];
+                col0 += widths[k];
                 pd.nch = (int32_t)ceil_div(pd.width, kChunk);
                 pd.slot_begin = pd.slot_end = 0;
                 if (td.rows > 0)
