@@ -10,14 +10,17 @@
 // Lane a of a group owns element a = i n + j (row-major vec(X), as the
 // oracle): its X_a, its momentum and row a of A in registers, plus its own
 // copies of R_i, C_j and 1^T R.  The gradient A vec(X) reads X from shared
-// memory with 128-bit broadcast loads.  [P^(1)]^2 is written twice:
-// row-major with rows padded to NB and column-major with columns padded to
-// MB (padding stays zero); a row sum and a column sum are then a few 128-bit
-// loads each, added in a fixed order, so the lanes of one row (column) hold
+// memory with 128-bit broadcast loads and accumulates with paired float32
+// FMAs (two round-to-nearest FMAs per instruction).  [P^(1)]^2 is written
+// twice: row-major with row stride RS and column-major with column stride CS
+// (NB and MB, plus 4 when that is a multiple of 8, so that consecutive rows
+// or columns start in different 16-byte bank groups; padding stays zero).
+// A row sum and a column sum are then a few 128-bit loads each, added in a
+// fixed order with paired adds, so the lanes of one row (column) hold
 // bit-identical R_i (C_j).  The total comes from an xor butterfly of
-// shuffles, which also leaves identical bits in every lane.  One warp barrier per step
-// (everything is exchanged together, double buffered); no global memory
-// inside the step loop but the recorded energies.
+// shuffles, which also leaves identical bits in every lane.  One warp barrier
+// per step (everything is exchanged together, double buffered); no global
+// memory inside the step loop but the recorded energies.
 
 // One step k follows the BACD sub-steps of the splitting table (Appendix A):
 //   B  P^(B)_k = P_k - h A vec(X_k)
