@@ -33,6 +33,20 @@
  *     are detected before any work is enqueued.  Errors of work already
  *     enqueued surface as RIKFAD_ERR_CUDA on a later call.
  *   - A handle is not thread-safe: calls on one handle must not overlap.
+ *   - Non-finite guard.  The friction of Eq. xi_def divides by 1^T R +
+ *     eps_stab and every element of a matrix reads R and C, so one
+ *     non-finite gradient or momentum element poisons its whole matrix
+ *     within a step (and, with the paper's GPT2-S setting mu = 1.36e-6, the
+ *     gain (1 - e^{-alpha h})/(mu alpha) ~ 7e4 amplifies any blow-up).  The
+ *     kernels therefore test every R_i and C_j they write, every partial sum
+ *     of 1^T R and every element-wise friction value; a non-finite one is
+ *     recorded on the device and in a page-locked host flag.  A non-finite
+ *     P^(1) always shows there (R_i sums its row's squares, C_j its
+ *     column's); a non-finite X alone (a caller-supplied one, with finite
+ *     momentum) does not.  Once a report is visible on the host, rikfad_step
+ *     returns RIKFAD_ERR_NONFINITE and enqueues nothing; rikfad_check_finite
+ *     waits, names the tensor and clears the report.  The check adds no
+ *     memory traffic.
  */
 #ifndef RIKFAD_H
 #define RIKFAD_H
@@ -57,6 +71,7 @@ enum rikfad_status {
     RIKFAD_ERR_ALIGN = -2, /* a pointer does not meet the documented alignment */
     RIKFAD_ERR_CUDA = -3,  /* a CUDA runtime call or an earlier kernel failed */
     RIKFAD_ERR_OOM = -4,   /* device or pinned host allocation failed */
+    RIKFAD_ERR_NONFINITE = -5, /* a step produced a non-finite factor, friction or 1^T R */
     RIKFAD_ERR_STATE = -6  /* call not valid for this handle (e.g. wrong device) */
 };
 
@@ -230,7 +245,9 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
 
 /* Read the friction denominators 1^T R of every matrix (ntensors floats, 0 for
  * element-wise tensors) into host memory, enqueued on `stream`; the values
- * are valid once the stream reaches this point (the call itself waits for it). */
+ * are valid once the stream reaches this point (the call itself waits for it).
+ * Returns RIKFAD_ERR_NONFINITE (after writing host_out) if a step reported a
+ * non-finite result; the report stays until rikfad_check_finite clears it. */
 RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *stream);
 
 /*
@@ -256,6 +273,18 @@ RIKFAD_API int rikfad_import_state(rikfad_handle h, const void *dev_src, void *s
 RIKFAD_API int rikfad_profile_enable(rikfad_handle h, int enable);
 RIKFAD_API int rikfad_profile_read(rikfad_handle h, double *step_kernel_ms,
                                    double *finalize_kernel_ms, int64_t *steps);
+
+/*
+ * Wait for the work enqueued on `stream` and report whether any step since
+ * the last clear produced a non-finite factor R_i, C_j, partial sum of 1^T R
+ * or element-wise friction value (the guard described at the top of this
+ * header).  Returns RIKFAD_OK, or RIKFAD_ERR_NONFINITE with the lowest
+ * offending tensor index in rikfad_last_error; in that case the report is
+ * cleared, so that rikfad_step accepts work again once the caller has
+ * restored a finite state (rikfad_import_state or rikfad_set_factors clear
+ * the report as well).  The non-finite values themselves stay in the state.
+ */
+RIKFAD_API int rikfad_check_finite(rikfad_handle h, void *stream);
 
 /* Number of kernel launches one rikfad_step enqueues for this handle. */
 RIKFAD_API int rikfad_launches_per_step(rikfad_handle h);
@@ -362,6 +391,32 @@ RIKFAD_API int rikfad_quadratic_run(int64_t batch, int64_t m, int64_t n, const f
                                     const rikfad_hparams *hp, int64_t nsteps,
                                     const int64_t *record, int64_t nrecord, float *energy,
                                     void *stream);
+
+/*
+ * Testing hooks.  These have no counterpart in the paper.
+ *
+ * rikfad_debug_check_failures: a library compiled with -DRIKFAD_CHECKED
+ * (librikfad_checked.so, built by build(checked=True)) verifies inside every
+ * kernel, before each access, that the plan's block, piece, tensor, panel,
+ * slot and finalise-item indices, the row, column and element ranges, the
+ * offsets into the factor, partial-sum and denominator buffers, and the
+ * pointer-table entries (non-NULL; 16-byte aligned on the 8-wide paths) lie
+ * within what the planner produced.  A failed check is counted and the
+ * access it guarded is skipped; nothing traps.  This call waits for the
+ * device and writes the number of failed checks since the handle was created
+ * to *count (and the code of the first, rikfad_checks.cuh, to *first_code);
+ * *count is -1 in a library built without the checks.
+ *
+ * rikfad_debug_fail_allocation(n): the n-th device or page-locked host
+ * allocation the library makes from now on (n >= 1, counted over all
+ * threads) reports failure as if memory were exhausted; n <= 0 turns this
+ * off.  It exercises the clean-up paths of rikfad_create without exhausting
+ * any memory.  rikfad_debug_live_allocations returns how many allocations the
+ * library currently holds (0 once every handle is destroyed).
+ */
+RIKFAD_API int rikfad_debug_check_failures(rikfad_handle h, int64_t *count, int *first_code);
+RIKFAD_API void rikfad_debug_fail_allocation(int64_t n);
+RIKFAD_API int64_t rikfad_debug_live_allocations(void);
 
 /* Last error message of the calling thread ("" if none). */
 RIKFAD_API const char *rikfad_last_error(void);

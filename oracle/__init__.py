@@ -32,7 +32,7 @@ def load(path):
     i64 = ctypes.c_int64
     dp = ctypes.POINTER(ctypes.c_double)
     d = ctypes.c_double
-    L.orc_step_matrix.argtypes = [i64, i64, dp, dp, dp, dp, dp, d, d, d, d, d, dp, dp]
+    L.orc_step_matrix.argtypes = [i64, i64, dp, dp, dp, dp, dp, d, d, d, d, d, dp, dp, dp]
     L.orc_step_matrix.restype = ctypes.c_int
     L.orc_step_vector.argtypes = [i64, dp, dp, dp, dp, d, d, d, d]
     L.orc_step_vector.restype = ctypes.c_int
@@ -68,16 +68,21 @@ class HParams:
         self.eps_stab = float(eps_stab)
 
 
-def step_matrix(X, P, R, C, G, h, hp):
-    """One BACD step (Appendix A table) for an m x n matrix, in place."""
+def step_matrix(X, P, R, C, G, h, hp, P1=None):
+    """One BACD step (Appendix A table) for an m x n matrix, in place.  If
+    ``P1`` (an m x n float64 array) is given it receives the half-damped
+    momentum P^(1) of sub-step C."""
     m, n = X.shape
     if P.shape != (m, n) or G.shape != (m, n) or R.shape != (m,) or C.shape != (n,):
+        raise ValueError("shape mismatch")
+    if P1 is not None and P1.shape != (m, n):
         raise ValueError("shape mismatch")
     rowsq = np.empty(max(m, 1))
     colsq = np.empty(n)
     rc = lib().orc_step_matrix(m, n, _f64(X, "X"), _f64(P, "P"), _f64(R, "R"), _f64(C, "C"),
                                _f64(G, "G"), float(h), hp.alpha, hp.mu, hp.gamma, hp.eps_stab,
-                               _f64(rowsq, "rowsq"), _f64(colsq, "colsq"))
+                               _f64(rowsq, "rowsq"), _f64(colsq, "colsq"),
+                               None if P1 is None else _f64(P1, "P1"))
     if rc != 0:
         raise ValueError("orc_step_matrix rejected its arguments")
 

@@ -20,8 +20,9 @@ def friction_tensor(R, C, eps_stab):
     return np.outer(R, C) / denom
 
 
-def step_matrix_explicit(X, P, R, C, G, h, alpha, mu, gamma, eps_stab):
-    """Return (X, P, R, C) after one BACD step; inputs are not modified."""
+def step_matrix_explicit(X, P, R, C, G, h, alpha, mu, gamma, eps_stab, return_p1=False):
+    """Return (X, P, R, C) after one BACD step (and P^(1), the half-damped
+    momentum of sub-step C, if ``return_p1``); inputs are not modified."""
     X = np.array(X, np.float64)
     P = np.array(P, np.float64)
     R = np.array(R, np.float64)
@@ -37,4 +38,6 @@ def step_matrix_explicit(X, P, R, C, G, h, alpha, mu, gamma, eps_stab):
     C = decay * C + gain * Q.sum(axis=0)                  # ([P1]^2)^T 1_m
     P2 = P1 * np.exp(-(h / 2) * friction_tensor(R, C, eps_stab))   # C, second half
     P = P2 * np.exp(-gamma * h)                           # D
+    if return_p1:
+        return X, P, R, C, P1
     return X, P, R, C

@@ -72,10 +72,12 @@ static double friction_entry(double Ri, double Cj, double denom)
  *   G     : m*n, the gradient grad f(X_n)
  *   h     : step size; alpha, mu, gamma, eps_stab: hyperparameters
  *   rowsq : scratch of m doubles, colsq: scratch of n doubles (caller-owned)
+ *   P1    : NULL, or m*n doubles that receive the half-damped momentum P^(1)
+ *           of sub-step C (an output only; nothing else depends on it)
  */
 int orc_step_matrix(int64_t m, int64_t n, double *X, double *P, double *R, double *C,
                     const double *G, double h, double alpha, double mu, double gamma,
-                    double eps_stab, double *rowsq, double *colsq)
+                    double eps_stab, double *rowsq, double *colsq, double *P1)
 {
     /* m = 0 is an empty matrix: no momentum, and C only decays. */
     if (m < 0 || n < 1 || !hparams_ok(h, alpha, mu, gamma, eps_stab))
@@ -97,6 +99,9 @@ int orc_step_matrix(int64_t m, int64_t n, double *X, double *P, double *R, doubl
     for (int64_t i = 0; i < m; ++i)
         for (int64_t j = 0; j < n; ++j)
             P[i * n + j] = P[i * n + j] * exp(-0.5 * h * friction_entry(R[i], C[j], denom));
+    if (P1 != 0)
+        for (int64_t k = 0; k < N; ++k)
+            P1[k] = P[k];
 
     /* Sub-step C, factor update with the momentum held at P^(1): the exact
      * solution over time h of dR/dt = [P]^2 1_n / mu - alpha R (and the same
@@ -235,7 +240,7 @@ int orc_dense_quadratic_run(int64_t m, int64_t n, const double *A, double *X, do
             G[a] = g;
         }
         int rc = orc_step_matrix(m, n, X, P, R, C, G, h, alpha, mu, gamma, eps_stab, rowsq,
-                                 colsq);
+                                 colsq, 0);
         if (rc != ORC_OK)
             return rc;
     }

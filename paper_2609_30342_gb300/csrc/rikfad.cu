@@ -2,6 +2,8 @@
 // argument checking, device state, and the launches of the step kernels.
 #include <cuda_runtime.h>
 
+#include <atomic>
+#include <climits>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -39,6 +41,70 @@ int cuda_fail(cudaError_t e, const char *what)
         if (e_ != cudaSuccess)                                \
             return cuda_fail(e_, what);                       \
     } while (0)
+
+// Every device and page-locked host allocation of the library goes through
+// these wrappers.  They count the allocations currently held (a leak check
+// for tests) and can be told to report the n-th allocation from now on as
+// failed (rikfad_debug_fail_allocation), which exercises the clean-up paths
+// without exhausting any memory.
+std::atomic<int64_t> g_fail_at{0};
+std::atomic<int64_t> g_alloc_calls{0};
+std::atomic<int64_t> g_live_allocs{0};
+
+bool injected_failure()
+{
+    const int64_t n = g_fail_at.load();
+    return n > 0 && g_alloc_calls.fetch_add(1) + 1 == n;
+}
+
+cudaError_t rk_malloc(void **p, size_t nb)
+{
+    *p = nullptr;
+    if (injected_failure())
+        return cudaErrorMemoryAllocation;
+    const cudaError_t e = cudaMalloc(p, nb);
+    if (e == cudaSuccess)
+        ++g_live_allocs;
+    else
+        *p = nullptr;
+    return e;
+}
+
+cudaError_t rk_malloc_host(void **p, size_t nb, unsigned flags)
+{
+    *p = nullptr;
+    if (injected_failure())
+        return cudaErrorMemoryAllocation;
+    const cudaError_t e = cudaHostAlloc(p, nb, flags);
+    if (e == cudaSuccess)
+        ++g_live_allocs;
+    else
+        *p = nullptr;
+    return e;
+}
+
+void rk_free(void *p)
+{
+    if (p) {
+        cudaFree(p);
+        --g_live_allocs;
+    }
+}
+
+void rk_free_host(void *p)
+{
+    if (p) {
+        cudaFreeHost(p);
+        --g_live_allocs;
+    }
+}
+
+int alloc_fail(cudaError_t e, const char *what)
+{
+    if (e == cudaErrorMemoryAllocation)
+        return fail(RIKFAD_ERR_OOM, std::string(what) + " failed: out of memory");
+    return cuda_fail(e, what);
+}
 
 constexpr uint64_t kImageTag = 0x31444146694b5221ull;   // "!RKiFAD1"
 constexpr size_t kImageHeader = 64;
@@ -96,6 +162,10 @@ struct rikfad_handle_s {
     float *d_spart = nullptr;
     float *d_den = nullptr;
     float *h_den = nullptr;         // pinned
+    int32_t *d_guard = nullptr;     // lowest tensor with a non-finite result (INT32_MAX: none)
+    int32_t *h_guard = nullptr;     // mapped page-locked host flag, set by the kernels
+    int32_t *h_guard_dev = nullptr; // its device address
+    int32_t *d_checks = nullptr;    // failed device checks: count, first code (checked builds)
     size_t workspace = 0;
 
     PtrTable step_ptrs;             // x | grad | p
@@ -106,8 +176,8 @@ struct rikfad_handle_s {
     float *d_diag_u = nullptr, *d_diag_v = nullptr, *d_diag_w = nullptr, *d_diag_wpart = nullptr;
     double *d_diag_norms = nullptr;
 
-    // in-order ("sweep") schedule
-    bool sweep = true;
+    // in-order ("sweep") schedule, allocated only when selected
+    bool sweep = false;
     int sweep_blocks = 0;
     UnitDev *d_units = nullptr;
     NodeDev *d_nodes = nullptr;
@@ -145,10 +215,9 @@ int upload(T **dst, const std::vector<T> &src, size_t &bytes)
     if (src.empty())
         return RIKFAD_OK;
     const size_t nb = src.size() * sizeof(T);
-    cudaError_t e = cudaMalloc((void **)dst, nb);
+    cudaError_t e = rk_malloc((void **)dst, nb);
     if (e != cudaSuccess)
-        return e == cudaErrorMemoryAllocation ? fail(RIKFAD_ERR_OOM, "cudaMalloc of a plan table failed")
-                                              : cuda_fail(e, "cudaMalloc");
+        return alloc_fail(e, "cudaMalloc of a plan table");
     bytes += nb;
     RK_CUDA(cudaMemcpy(*dst, src.data(), nb, cudaMemcpyHostToDevice), "cudaMemcpy plan table");
     return RIKFAD_OK;
@@ -160,10 +229,9 @@ int alloc_zero(float **dst, int64_t floats, size_t &bytes)
     if (floats <= 0)
         return RIKFAD_OK;
     const size_t nb = (size_t)floats * sizeof(float);
-    cudaError_t e = cudaMalloc((void **)dst, nb);
+    cudaError_t e = rk_malloc((void **)dst, nb);
     if (e != cudaSuccess)
-        return e == cudaErrorMemoryAllocation ? fail(RIKFAD_ERR_OOM, "cudaMalloc failed")
-                                              : cuda_fail(e, "cudaMalloc");
+        return alloc_fail(e, "cudaMalloc");
     bytes += nb;
     RK_CUDA(cudaMemset(*dst, 0, nb), "cudaMemset");
     return RIKFAD_OK;
@@ -176,23 +244,21 @@ int ptrtable_init(PtrTable &t, int count, size_t &bytes)
     t.valid = false;
     if (count == 0)
         return RIKFAD_OK;
-    cudaError_t e = cudaMalloc((void **)&t.dev, sizeof(void *) * count);
+    cudaError_t e = rk_malloc((void **)&t.dev, sizeof(void *) * count);
     if (e != cudaSuccess)
-        return fail(RIKFAD_ERR_OOM, "cudaMalloc of the pointer table failed");
+        return alloc_fail(e, "cudaMalloc of the pointer table");
     bytes += sizeof(void *) * count;
-    e = cudaMallocHost((void **)&t.pinned, sizeof(void *) * count);
+    e = rk_malloc_host((void **)&t.pinned, sizeof(void *) * count, cudaHostAllocDefault);
     if (e != cudaSuccess)
-        return fail(RIKFAD_ERR_OOM, "cudaMallocHost of the pointer staging failed");
+        return alloc_fail(e, "cudaHostAlloc of the pointer staging");
     RK_CUDA(cudaEventCreateWithFlags(&t.uploaded, cudaEventDisableTiming), "cudaEventCreate");
     return RIKFAD_OK;
 }
 
 void ptrtable_free(PtrTable &t)
 {
-    if (t.dev)
-        cudaFree(t.dev);
-    if (t.pinned)
-        cudaFreeHost(t.pinned);
+    rk_free(t.dev);
+    rk_free_host(t.pinned);
     if (t.uploaded)
         cudaEventDestroy(t.uploaded);
     t = PtrTable();
@@ -237,30 +303,15 @@ bool hparams_ok(const rikfad_hparams &hp, std::string &why)
 
 void release(rikfad_handle h)
 {
-    cudaFree(h->d_tensors);
-    cudaFree(h->d_panels);
-    cudaFree(h->d_pieces);
-    cudaFree(h->d_block_piece);
-    cudaFree(h->d_slot_off);
-    cudaFree(h->d_fin);
-    cudaFree(h->d_fac);
-    cudaFree(h->d_rowpart);
-    cudaFree(h->d_colpart);
-    cudaFree(h->d_spart);
-    cudaFree(h->d_den);
-    cudaFree(h->d_diag_u);
-    cudaFree(h->d_diag_v);
-    cudaFree(h->d_diag_w);
-    cudaFree(h->d_diag_wpart);
-    cudaFree(h->d_diag_norms);
-    cudaFree(h->d_units);
-    cudaFree(h->d_nodes);
-    cudaFree(h->d_trees);
-    cudaFree(h->d_partials);
-    cudaFree(h->d_counts);
-    cudaFree(h->d_fetch);
-    if (h->h_den)
-        cudaFreeHost(h->h_den);
+    for (void *p : {(void *)h->d_tensors, (void *)h->d_panels, (void *)h->d_pieces, (void *)h->d_block_piece,
+                    (void *)h->d_slot_off, (void *)h->d_fin, (void *)h->d_fac, (void *)h->d_rowpart,
+                    (void *)h->d_colpart, (void *)h->d_spart, (void *)h->d_den, (void *)h->d_guard,
+                    (void *)h->d_checks, (void *)h->d_diag_u, (void *)h->d_diag_v, (void *)h->d_diag_w,
+                    (void *)h->d_diag_wpart, (void *)h->d_diag_norms, (void *)h->d_units, (void *)h->d_nodes,
+                    (void *)h->d_trees, (void *)h->d_partials, (void *)h->d_counts, (void *)h->d_fetch})
+        rk_free(p);
+    rk_free_host(h->h_den);
+    rk_free_host(h->h_guard);
     ptrtable_free(h->step_ptrs);
     ptrtable_free(h->canon_ptrs);
     for (cudaEvent_t ev : h->prof_events)
@@ -317,6 +368,55 @@ void launch_sweep(const StepParams &p, const SweepParams &sp, bool reuse, int nb
         rikfad_sweep_kernel<GT, false><<<nblocks, kThreads, 0, s>>>(p, sp);
 }
 
+CheckBounds bounds(const rikfad_handle h)
+{
+    const Plan &p = h->plan;
+    CheckBounds cb{};
+    cb.ntensors = (int32_t)p.tensors.size();
+    cb.npanels = (int32_t)p.panels.size();
+    cb.npieces = (int32_t)p.pieces.size();
+    cb.nblocks = p.nblocks;
+    cb.nfin = (int32_t)p.fin_items.size();
+    cb.nslots = (int32_t)p.slot_off.size();
+    cb.fac_floats = p.fac_floats;
+    cb.rowpart_floats = p.rowpart_floats;
+    cb.colpart_floats = p.colpart_floats;
+    cb.spart_floats = p.spart_floats;
+    cb.errors = h->d_checks;
+    return cb;
+}
+
+Guard guard(const rikfad_handle h) { return Guard{h->d_guard, h->h_guard_dev}; }
+
+// Forget an earlier non-finite report (the device word and the host flag);
+// stream-ordered for the device word.
+int clear_guard(rikfad_handle h, cudaStream_t stream)
+{
+    static const int32_t none = INT32_MAX;
+    RK_CUDA(cudaMemcpyAsync(h->d_guard, &none, sizeof none, cudaMemcpyHostToDevice, stream),
+            "cudaMemcpyAsync guard");
+    RK_CUDA(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+    *(volatile int32_t *)h->h_guard = 0;
+    return RIKFAD_OK;
+}
+
+// RIKFAD_ERR_NONFINITE naming the offending tensor, if the kernels reported
+// one (call after the work has completed).
+int nonfinite_status(rikfad_handle h, cudaStream_t stream)
+{
+    if (*(volatile int32_t *)h->h_guard == 0)
+        return RIKFAD_OK;
+    int32_t first = INT32_MAX;
+    RK_CUDA(cudaMemcpyAsync(&first, h->d_guard, sizeof first, cudaMemcpyDeviceToHost, stream),
+            "cudaMemcpyAsync guard");
+    RK_CUDA(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+    return fail(RIKFAD_ERR_NONFINITE,
+                "a step produced a non-finite factor, friction or denominator (first tensor: " +
+                    (first == INT32_MAX ? std::string("unknown") : std::to_string(first)) +
+                    "); restore the state (rikfad_import_state, rikfad_set_factors) and call "
+                    "rikfad_check_finite to clear the report");
+}
+
 int finalize(rikfad_handle h, float decay, float gain, int resum_only, cudaStream_t stream)
 {
     if (h->plan.fin_items.empty())
@@ -333,6 +433,8 @@ int finalize(rikfad_handle h, float decay, float gain, int resum_only, cudaStrea
     f.decay = decay;
     f.gain = gain;
     f.resum_only = resum_only;
+    f.guard = guard(h);
+    f.chk = bounds(h);
     RK_CUDA(launch_pdl(rikfad_finalize_kernel, (int)h->plan.fin_items.size(), kFinThreads, stream, f),
             "launch rikfad_finalize_kernel");
     return RIKFAD_OK;
@@ -372,6 +474,7 @@ int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool 
         c.ex_prev = (float)(-0.5 * h->pending_step * M_LOG2E);
         c.damp_prev = (float)std::exp(-h->hp.gamma * h->pending_step);
         c.eps = (float)h->hp.eps_stab;
+        c.chk = bounds(h);
         RK_CUDA(launch_pdl(rikfad_canonical_kernel, h->plan.nblocks, kThreads, stream, c),
                 "launch rikfad_canonical_kernel");
     }
@@ -507,18 +610,25 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     }
     if (occ_min < 1)
         return fail(RIKFAD_ERR_CUDA, "step kernel cannot be resident on this device");
+    // Static schedule by default; RIKFAD_SCHEDULE=sweep selects the in-order
+    // one-kernel schedule (slower on GB300, see rikfad_sweep.cuh), whose
+    // units, trees and partials are built and allocated only then.
+    const char *env = std::getenv("RIKFAD_SCHEDULE");
+    const bool sweep = env && std::strcmp(env, "sweep") == 0 && !shadow;
     int occ_sweep = 1 << 30;
-    const void *sweep_kernels[4] = {(const void *)rikfad_sweep_kernel<float, true>,
-                                    (const void *)rikfad_sweep_kernel<float, false>,
-                                    (const void *)rikfad_sweep_kernel<__nv_bfloat16, true>,
-                                    (const void *)rikfad_sweep_kernel<__nv_bfloat16, false>};
-    for (const void *k : sweep_kernels) {
-        RK_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, 0),
-                "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
-        occ_sweep = std::min(occ_sweep, occ);
+    if (sweep) {
+        const void *sweep_kernels[4] = {(const void *)rikfad_sweep_kernel<float, true>,
+                                        (const void *)rikfad_sweep_kernel<float, false>,
+                                        (const void *)rikfad_sweep_kernel<__nv_bfloat16, true>,
+                                        (const void *)rikfad_sweep_kernel<__nv_bfloat16, false>};
+        for (const void *k : sweep_kernels) {
+            RK_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, 0),
+                    "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+            occ_sweep = std::min(occ_sweep, occ);
+        }
+        if (occ_sweep < 1)
+            return fail(RIKFAD_ERR_CUDA, "sweep kernel cannot be resident on this device");
     }
-    if (occ_sweep < 1)
-        return fail(RIKFAD_ERR_CUDA, "sweep kernel cannot be resident on this device");
 
     rikfad_handle h = new rikfad_handle_s();
     h->device = dev;
@@ -533,14 +643,11 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
         delete h;
         return fail(RIKFAD_ERR_ARG, why);
     }
-    build_sweep(shapes, ntensors, h->plan);
-    {
-        // Static schedule by default; RIKFAD_SCHEDULE=sweep selects the
-        // in-order one-kernel schedule (slower on GB300, see rikfad_sweep.cuh).
-        const char *env = std::getenv("RIKFAD_SCHEDULE");
-        h->sweep = env && std::strcmp(env, "sweep") == 0 && !shadow;
+    h->sweep = sweep;
+    if (sweep) {
+        build_sweep(shapes, ntensors, h->plan);
+        h->sweep_blocks = sms * occ_sweep;
     }
-    h->sweep_blocks = sms * occ_sweep;
     const Plan &p = h->plan;
     size_t ws = 0;
     int rc = RIKFAD_OK;
@@ -556,14 +663,31 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     if (!rc) rc = alloc_zero(&h->d_colpart, p.colpart_floats, ws);
     if (!rc) rc = alloc_zero(&h->d_spart, p.spart_floats, ws);
     if (!rc) rc = alloc_zero(&h->d_den, std::max(ntensors, 1), ws);
-    if (!rc && cudaMallocHost((void **)&h->h_den, sizeof(float) * std::max(ntensors, 1)) != cudaSuccess)
-        rc = fail(RIKFAD_ERR_OOM, "cudaMallocHost failed");
-    if (!rc) rc = upload(&h->d_units, p.units, ws);
-    if (!rc) rc = upload(&h->d_nodes, p.nodes, ws);
-    if (!rc) rc = upload(&h->d_trees, p.trees, ws);
-    if (!rc) rc = alloc_zero(&h->d_partials, p.partial_floats, ws);
-    if (!rc) rc = alloc_zero((float **)&h->d_counts, (int64_t)p.nodes.size() + ntensors + 1, ws);
-    if (!rc) rc = alloc_zero((float **)&h->d_fetch, 4, ws);
+    if (!rc) {
+        cudaError_t e = rk_malloc_host((void **)&h->h_den, sizeof(float) * std::max(ntensors, 1),
+                                       cudaHostAllocDefault);
+        if (e != cudaSuccess)
+            rc = alloc_fail(e, "cudaHostAlloc of the denominator read-back");
+    }
+    // Non-finite guard: a device word (lowest offending tensor) and a mapped
+    // host flag the kernels set, so rikfad_step sees a report without waiting.
+    if (!rc) rc = alloc_zero((float **)&h->d_guard, 1, ws);
+    if (!rc) {
+        cudaError_t e = rk_malloc_host((void **)&h->h_guard, sizeof(int32_t), cudaHostAllocMapped);
+        if (e != cudaSuccess)
+            rc = alloc_fail(e, "cudaHostAlloc of the non-finite flag");
+        else if ((e = cudaHostGetDevicePointer((void **)&h->h_guard_dev, h->h_guard, 0)) != cudaSuccess)
+            rc = cuda_fail(e, "cudaHostGetDevicePointer");
+    }
+    if (!rc) rc = alloc_zero((float **)&h->d_checks, 2, ws);
+    if (!rc && sweep) {
+        rc = upload(&h->d_units, p.units, ws);
+        if (!rc) rc = upload(&h->d_nodes, p.nodes, ws);
+        if (!rc) rc = upload(&h->d_trees, p.trees, ws);
+        if (!rc) rc = alloc_zero(&h->d_partials, p.partial_floats, ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_counts, (int64_t)p.nodes.size() + ntensors + 1, ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_fetch, 4, ws);
+    }
     if (!rc && shadow) {
         int64_t max_m = 1, max_n = 1, max_parts = 1;
         for (const TensorDev &td : p.tensors)
@@ -580,6 +704,7 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     }
     if (!rc) rc = ptrtable_init(h->step_ptrs, 3 * ntensors, ws);
     if (!rc) rc = ptrtable_init(h->canon_ptrs, 2 * ntensors, ws);
+    if (!rc) rc = clear_guard(h, 0);
     if (!rc) {
         cudaError_t e = cudaDeviceSynchronize();
         if (e != cudaSuccess)
@@ -626,6 +751,12 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
     const int T = h->ntensors;
     if (T > 0 && (x == nullptr || grad == nullptr || p == nullptr))
         return fail(RIKFAD_ERR_ARG, "pointer array is NULL");
+    // A non-finite result reported by an earlier step (seen without waiting):
+    // nothing more is enqueued until the report is cleared.
+    if (*(volatile int32_t *)h->h_guard != 0)
+        return fail(RIKFAD_ERR_NONFINITE, "an earlier step produced a non-finite factor, friction or "
+                                          "denominator; rikfad_check_finite names the tensor and clears "
+                                          "the report");
     const double decay_d = std::exp(-h->hp.alpha * step);
     const double gain_d = std::isinf(h->hp.mu) ? 0.0 : -std::expm1(-h->hp.alpha * step) / (h->hp.mu * h->hp.alpha);
     if (!std::isfinite((float)gain_d))
@@ -692,6 +823,8 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
         a.decay = (float)decay_d;
         a.gain = (float)gain_d;
         a.eps = (float)h->hp.eps_stab;
+        a.guard = guard(h);
+        a.chk = bounds(h);
         const bool reuse = (step == h->pending_step);
         if (h->sweep) {
             SweepParams sp{};
@@ -803,6 +936,9 @@ RIKFAD_API int rikfad_set_factors(rikfad_handle h, int t, const float *R_host, c
         if (!(std::isfinite(C_host[j]) && C_host[j] >= 0))
             return fail(RIKFAD_ERR_ARG, "factor values must be finite and >= 0");
     RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    rc = clear_guard(h, 0);
+    if (rc)
+        return rc;
     if (R_host && nr > 0)
         RK_CUDA(cudaMemcpy(h->d_fac + td.fac_off, R_host, sizeof(float) * nr, cudaMemcpyHostToDevice),
                 "cudaMemcpy factors");
@@ -827,7 +963,7 @@ RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *
     if (T == 0)
         return RIKFAD_OK;
     cudaStream_t s = (cudaStream_t)stream;
-    DenParams d{h->d_tensors, h->d_spart, h->d_den, T};
+    DenParams d{h->d_tensors, h->d_spart, h->d_den, T, bounds(h)};
     const int warps = 8;
     rikfad_denominators_kernel<<<(T + warps - 1) / warps, 32 * warps, 0, s>>>(d);
     RK_CUDA(cudaGetLastError(), "launch rikfad_denominators_kernel");
@@ -835,7 +971,7 @@ RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *
             "cudaMemcpyAsync denominators");
     RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
     std::memcpy(host_out, h->h_den, sizeof(float) * T);
-    return RIKFAD_OK;
+    return nonfinite_status(h, s);
 }
 
 RIKFAD_API size_t rikfad_state_image_bytes(rikfad_handle h)
@@ -892,6 +1028,9 @@ RIKFAD_API int rikfad_import_state(rikfad_handle h, const void *dev_src, void *s
     if (hd.alpha != h->hp.alpha || hd.mu != h->hp.mu || hd.gamma != h->hp.gamma ||
         hd.eps_stab != h->hp.eps_stab)
         return fail(RIKFAD_ERR_ARG, "state image was exported with other hyperparameters");
+    rc = clear_guard(h, s);
+    if (rc)
+        return rc;
     if (h->plan.fac_floats > 0)
         RK_CUDA(cudaMemcpyAsync(h->d_fac, (const char *)dev_src + kImageHeader,
                                 sizeof(float) * h->plan.fac_floats, cudaMemcpyDeviceToDevice, s),
@@ -997,7 +1136,7 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     const float *R = h->d_fac + td.fac_off;
     const float *C = h->d_fac + td.fac_off + m;
     // 1^T R exactly as the step kernels form it
-    DenParams d{h->d_tensors, h->d_spart, h->d_den, h->ntensors};
+    DenParams d{h->d_tensors, h->d_spart, h->d_den, h->ntensors, bounds(h)};
     rikfad_denominators_kernel<<<(h->ntensors + kWarps - 1) / kWarps, kThreads, 0, s>>>(d);
     RK_CUDA(cudaGetLastError(), "launch rikfad_denominators_kernel");
     float den_sum = 0.f;
@@ -1071,5 +1210,55 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     out[5] = (double)std::min(it, max_iters);
     return RIKFAD_OK;
 }
+
+RIKFAD_API int rikfad_check_finite(rikfad_handle h, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    rc = nonfinite_status(h, s);
+    if (rc == RIKFAD_ERR_NONFINITE) {
+        const std::string msg = g_last_error;
+        const int rc2 = clear_guard(h, s);
+        if (rc2)
+            return rc2;
+        g_last_error = msg;
+    }
+    return rc;
+}
+
+RIKFAD_API int rikfad_debug_check_failures(rikfad_handle h, int64_t *count, int *first_code)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+#ifdef RIKFAD_CHECKED
+    int32_t w[2] = {0, 0};
+    RK_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    RK_CUDA(cudaMemcpy(w, h->d_checks, sizeof w, cudaMemcpyDeviceToHost), "cudaMemcpy check counters");
+    if (count)
+        *count = w[0];
+    if (first_code)
+        *first_code = w[1];
+#else
+    if (count)
+        *count = -1;
+    if (first_code)
+        *first_code = 0;
+#endif
+    return RIKFAD_OK;
+}
+
+RIKFAD_API void rikfad_debug_fail_allocation(int64_t n)
+{
+    g_fail_at.store(0);
+    g_alloc_calls.store(0);
+    g_fail_at.store(n > 0 ? n : 0);
+}
+
+RIKFAD_API int64_t rikfad_debug_live_allocations(void) { return g_live_allocs.load(); }
+
 
 }  // extern "C"

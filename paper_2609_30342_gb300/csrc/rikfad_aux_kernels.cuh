@@ -11,6 +11,7 @@ struct DenParams {
     const float *spart;
     float *out;
     int ntensors;
+    CheckBounds chk;           // read by checked builds only
 };
 
 struct CanonParams {
@@ -25,6 +26,7 @@ struct CanonParams {
     float ex_prev;
     float damp_prev;
     float eps;
+    CheckBounds chk;           // read by checked builds only
 };
 
 struct FinParams {
@@ -39,7 +41,44 @@ struct FinParams {
     float decay;
     float gain;
     int resum_only;            // 1: only recompute the partial sums of R
+    Guard guard;
+    CheckBounds chk;           // read by checked builds only
 };
+
+// Checks of one finalise item (checked builds): its tensor, rows or panel
+// and slots, and the offsets they lead to.
+__device__ __forceinline__ bool fin_item_ok(const FinParams &f, const FinItemDev &it, const TensorDev &td)
+{
+    (void)f; (void)it; (void)td;
+    const CheckBounds &cb = f.chk;
+    (void)cb;
+    if (!RK_DEV_CHECK(cb, td.cols > 0 && td.fac_off >= 0 && td.fac_off + td.rows + td.cols <= cb.fac_floats,
+                      kChkFactors))
+        return false;
+    if (it.kind == kFinRows)
+        return RK_DEV_CHECK(cb, it.begin >= 0 && it.begin <= it.end && it.end <= td.rows, kChkRows) &&
+               RK_DEV_CHECK(cb, it.chunk >= 0 && it.chunk < td.spart_cnt && td.spart_off >= 0 &&
+                                    (int64_t)td.spart_off + td.spart_cnt <= cb.spart_floats, kChkSpart) &&
+               RK_DEV_CHECK(cb, f.resum_only || (td.rowpart_off >= 0 &&
+                                    td.rowpart_off + (int64_t)td.npanels * td.rows <= cb.rowpart_floats),
+                            kChkRowpart);
+    if (!RK_DEV_CHECK(cb, it.kind == kFinCols, kChkKind) ||
+        !RK_DEV_CHECK(cb, it.panel >= td.panel0 && it.panel < td.panel0 + td.npanels && it.panel >= 0 &&
+                              it.panel < cb.npanels, kChkPanel))
+        return false;
+    if (f.resum_only)
+        return true;
+    const PanelDev pd = f.panels[it.panel];
+    const int ns = pd.slot_end - pd.slot_begin;
+    return RK_DEV_CHECK(cb, pd.tensor == it.tensor && pd.col0 >= 0 &&
+                                (int64_t)pd.col0 + pd.width <= td.cols, kChkCols) &&
+           RK_DEV_CHECK(cb, it.begin >= 0 && it.begin <= it.end && it.end <= pd.width, kChkCols) &&
+           RK_DEV_CHECK(cb, pd.slot_begin >= 0 && ns >= 0 && pd.slot_end <= cb.nslots &&
+                                (it.chunk != 0 || ns <= kFinSplitSlots), kChkColpart) &&
+           RK_DEV_CHECK(cb, ns == 0 || (f.slot_off[pd.slot_begin] >= 0 &&
+                                        f.slot_off[pd.slot_begin] + (int64_t)ns * pd.width <= cb.colpart_floats),
+                        kChkColpart);
+}
 
 
 // ---------------------------------------------------- finalise kernel
@@ -58,10 +97,16 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
 {
     __shared__ float wsum[kFinThreads / 32];
     __shared__ float csum[kFinThreads / 32][32];
+    if (!RK_DEV_CHECK(f.chk, (int)blockIdx.x < f.chk.nfin, kChkFinItem))
+        return;
     const FinItemDev it = f.items[blockIdx.x];
+    if (!RK_DEV_CHECK(f.chk, it.tensor >= 0 && it.tensor < f.chk.ntensors, kChkTensor))
+        return;
     const TensorDev td = f.tensors[it.tensor];
     wait_for_predecessor();
     allow_successor_launch();
+    if (!fin_item_ok(f, it, td))
+        return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (it.kind == kFinRows) {
         const int64_t i = it.begin + threadIdx.x;
@@ -79,6 +124,8 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
                 val = fmaf(f.gain, acc, f.decay * R[i]);
                 R[i] = val;
             }
+            if (!isfinite(val))
+                report_nonfinite(f.guard, it.tensor);
         }
         val = warp_sum(val);
         if (lane == 0)
@@ -87,8 +134,11 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
         if (threadIdx.x < 32) {
             float v = threadIdx.x < kFinThreads / 32 ? wsum[threadIdx.x] : 0.f;
             v = warp_sum(v);
-            if (threadIdx.x == 0)
+            if (threadIdx.x == 0) {
                 f.spart[td.spart_off + it.chunk] = v;
+                if (!isfinite(v))       // finite R whose sum overflows
+                    report_nonfinite(f.guard, it.tensor);
+            }
         }
     } else if (!f.resum_only && it.chunk == 0) {
         // A panel's slots are consecutive in colpart, pd.width apart (the
@@ -109,7 +159,10 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
                 if (u < ns)
                     acc += v[u];
             float *C = f.fac + td.fac_off + td.rows + pd.col0;
-            C[c] = fmaf(f.gain, acc, f.decay * C[c]);
+            const float cn = fmaf(f.gain, acc, f.decay * C[c]);
+            C[c] = cn;
+            if (!isfinite(cn))
+                report_nonfinite(f.guard, it.tensor);
         }
     } else if (!f.resum_only) {
         const PanelDev pd = f.panels[it.panel];
@@ -129,7 +182,10 @@ __global__ void __launch_bounds__(kFinThreads) rikfad_finalize_kernel(FinParams 
             for (int k = 0; k < kFinThreads / 32; ++k)
                 t += csum[k][lane];
             float *C = f.fac + td.fac_off + td.rows + pd.col0;
-            C[c] = fmaf(f.gain, t, f.decay * C[c]);
+            const float cn = fmaf(f.gain, t, f.decay * C[c]);
+            C[c] = cn;
+            if (!isfinite(cn))
+                report_nonfinite(f.guard, it.tensor);
         }
     }
 }
@@ -145,19 +201,29 @@ __global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     wait_for_predecessor();
     allow_successor_launch();
+    if (!RK_DEV_CHECK(c.chk, (int)blockIdx.x < c.chk.nblocks, kChkBlock))
+        return;
     const int q0 = c.block_piece[blockIdx.x], q1 = c.block_piece[blockIdx.x + 1];
+    if (!block_ok(c.chk, blockIdx.x, q0, q1))
+        return;
     for (int q = q0; q < q1; ++q) {
         const PieceDev pc = c.pieces[q];
+        if (!piece_tensor_ok(c.chk, pc))
+            continue;
         const TensorDev td = c.tensors[pc.tensor];
         const float *S = c.src[pc.tensor];
         float *D = c.dst[pc.tensor];
         if (pc.kind == kElements) {
-            if (S != D)
+            if (S != D && vector_piece_ok(c.chk, pc, td, D, nullptr, S, false))
                 for (int64_t e = pc.begin + threadIdx.x; e < pc.end; e += kThreads)
                     D[e] = S[e];
             continue;
         }
+        if (!piece_panel_ok(c.chk, pc, td))
+            continue;
         const PanelDev pd = c.panels[pc.panel];
+        if (!matrix_piece_ok(c.chk, pc, td, pd, D, nullptr, S, false))
+            continue;
         if (td.full) {      // element-wise friction: P already holds P_{n+1}
             if (S != D)
                 for (int64_t row = pc.begin + warp; row < pc.end; row += kWarps)
@@ -215,6 +281,9 @@ __global__ void rikfad_denominators_kernel(DenParams d)
     if (t >= d.ntensors)
         return;
     const TensorDev td = d.tensors[t];
+    if (!RK_DEV_CHECK(d.chk, td.spart_off >= 0 && (int64_t)td.spart_off + td.spart_cnt <= d.chk.spart_floats,
+                      kChkSpart))
+        return;
     const float s = td.cols == 0 ? 0.f : row_total(d.spart, td);
     if ((threadIdx.x & 31) == 0)
         d.out[t] = s;

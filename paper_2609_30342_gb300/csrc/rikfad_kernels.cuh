@@ -27,9 +27,25 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "rikfad_checks.cuh"
 #include "rikfad_plan.hpp"
 
 namespace rikfad {
+
+// Non-finite guard.  A kernel that produces a non-finite factor, friction or
+// denominator records the tensor: the lowest such index in device memory
+// (atomicMin; INT32_MAX when there is none) and a flag in page-locked host
+// memory that the host reads without waiting for the device.
+struct Guard {
+    int32_t *first;
+    volatile int32_t *host;
+};
+
+__device__ __forceinline__ void report_nonfinite(const Guard &g, int tensor)
+{
+    atomicMin(g.first, tensor);
+    *g.host = 1;
+}
 
 struct StepParams {
     const TensorDev *tensors;
@@ -51,6 +67,8 @@ struct StepParams {
     float decay;               // e^{-alpha h}
     float gain;                // (1 - e^{-alpha h})/(mu alpha)
     float eps;                 // eps_stab
+    Guard guard;
+    CheckBounds chk;           // read by checked builds only
 };
 
 // ---------------------------------------------------------------- helpers
@@ -334,6 +352,7 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
     float *XI = a.fac + td.fac_off;
     const int64_t b0 = pc.begin;                // multiple of 8 (planner)
     const int64_t nvec = (pc.end - b0) / 8;
+    bool bad = false;
     for (int64_t v = threadIdx.x; v < nvec; v += kThreads) {
         const int64_t e0 = b0 + v * 8;
         Grad8<GT> g;
@@ -343,8 +362,10 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
         load8(P + e0, p);
         load8(XI + e0, xi);
 #pragma unroll
-        for (int e = 0; e < 8; ++e)
+        for (int e = 0; e < 8; ++e) {
             vector_element(x[e], p[e], xi[e], g.get(e), a);
+            bad |= !isfinite(xi[e]);
+        }
         store8(X + e0, x);
         store8(P + e0, p);
         store8(XI + e0, xi);
@@ -352,10 +373,15 @@ __device__ __forceinline__ void vector_piece(const StepParams &a, const PieceDev
     for (int64_t e = b0 + nvec * 8 + threadIdx.x; e < pc.end; e += kThreads) {
         float x = X[e], p = P[e], xi = XI[e];
         vector_element(x, p, xi, grad_at(G, e), a);
+        bad |= !isfinite(xi);
         X[e] = x;
         P[e] = p;
         XI[e] = xi;
     }
+    // The friction is d xi + k [P^(1)]^2: non-finite exactly when the
+    // half-damped momentum (or the friction before) is.
+    if (bad)
+        report_nonfinite(a.guard, pc.tensor);
 }
 
 // ------------------------------ matrix with element-wise friction (full iKFAD)
@@ -481,17 +507,32 @@ __global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS) rikfad_step_
     __shared__ __align__(16) float Cs[kPanelMax];
     __shared__ __align__(16) float red[kWarps * kPanelMax];
     const int b = blockIdx.x;
+    if (!RK_DEV_CHECK(a.chk, b < a.chk.nblocks, kChkBlock))
+        return;
     const int q0 = a.block_piece[b], q1 = a.block_piece[b + 1];
     wait_for_predecessor();
     allow_successor_launch();
+    if (!block_ok(a.chk, b, q0, q1))
+        return;
     for (int q = q0; q < q1; ++q) {
         const PieceDev pc = a.pieces[q];
+        if (!piece_tensor_ok(a.chk, pc))
+            continue;
         const TensorDev td = a.tensors[pc.tensor];
         if (pc.kind == kElements) {
-            vector_piece<GT>(a, pc, td);
+            if (vector_piece_ok(a.chk, pc, td, a.xptr[pc.tensor], a.gptr[pc.tensor], a.pptr[pc.tensor],
+                                true))
+                vector_piece<GT>(a, pc, td);
             continue;
         }
+        if (!piece_panel_ok(a.chk, pc, td))
+            continue;
         const PanelDev pd = a.panels[pc.panel];
+        // Block-uniform: every thread evaluates the same checks on the same
+        // entries, so a skipped piece is skipped by the whole block.
+        if (!matrix_piece_ok(a.chk, pc, td, pd, a.xptr[pc.tensor], a.gptr[pc.tensor], a.pptr[pc.tensor],
+                             true))
+            continue;
         const int w = pd.width;
         // Stage this panel's C, clear the column accumulators.
         const float *C = a.fac + td.fac_off + td.rows + pd.col0;

@@ -75,6 +75,24 @@ struct FinItemDev {
     int64_t end;
 };
 
+// Extents every plan index and offset must stay within.  Kernels of a build
+// with RIKFAD_CHECKED verify each index against these before using it; a
+// failed check is counted in errors[0] (errors[1] keeps the code of the
+// first) and the access it guarded is skipped.  Other builds never read them.
+struct CheckBounds {
+    int32_t ntensors;
+    int32_t npanels;
+    int32_t npieces;
+    int32_t nblocks;
+    int32_t nfin;
+    int32_t nslots;
+    int64_t fac_floats;
+    int64_t rowpart_floats;
+    int64_t colpart_floats;
+    int64_t spart_floats;
+    int32_t *errors;
+};
+
 // ------------------------------------------------------------------------
 // In-order schedule ("sweep"): persistent blocks take small units of work
 // from a global counter in memory order, so the whole GPU streams through a

@@ -89,6 +89,8 @@ __device__ __forceinline__ void finish_tensor(const StepParams &a, const SweepPa
                 acc += __ldcg(rp + (int64_t)k * td.rows);
             val = fmaf(a.gain, acc, a.decay * R[i]);
             R[i] = val;
+            if (!isfinite(val))
+                report_nonfinite(a.guard, t);
         }
         val = warp_sum(val);
         if (lane == 0)
@@ -97,8 +99,11 @@ __device__ __forceinline__ void finish_tensor(const StepParams &a, const SweepPa
         if (tid < 32) {
             float v = tid < kWarps ? wsum[tid] : 0.f;
             v = warp_sum(v);
-            if (tid == 0)
+            if (tid == 0) {
                 s.spart[td.spart_off + ch] = v;
+                if (!isfinite(v))
+                    report_nonfinite(a.guard, t);
+            }
         }
         __syncthreads();
     }
@@ -108,7 +113,10 @@ __device__ __forceinline__ void finish_tensor(const StepParams &a, const SweepPa
         float *C = a.fac + td.fac_off + td.rows + pd.col0;
         for (int c = tid; c < pd.width; c += kThreads) {
             const float sum = td.rows > 0 ? __ldcg(s.partials + tr.root_off + c) : 0.f;
-            C[c] = fmaf(a.gain, sum, a.decay * C[c]);
+            const float cn = fmaf(a.gain, sum, a.decay * C[c]);
+            C[c] = cn;
+            if (!isfinite(cn))
+                report_nonfinite(a.guard, t);
         }
         if (td.rows > 0) {
             __syncthreads();

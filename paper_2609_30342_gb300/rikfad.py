@@ -12,13 +12,16 @@ import os
 import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "librikfad.so")
+# RIKFAD_LIBRARY may name another build of the same library (the checked
+# build, librikfad_checked.so); it is read when the library is first loaded.
+LIB_PATH = os.environ.get("RIKFAD_LIBRARY") or os.path.join(_PKG, "librikfad.so")
 
 OK = 0
 ERR_ARG = -1
 ERR_ALIGN = -2
 ERR_CUDA = -3
 ERR_OOM = -4
+ERR_NONFINITE = -5
 ERR_STATE = -6
 GRAD_F32 = 0
 GRAD_BF16 = 1
@@ -75,6 +78,11 @@ SIGNATURES = [
                                            ctypes.POINTER(ctypes.c_double),
                                            ctypes.POINTER(ctypes.c_int64)]),
     ("rikfad_launches_per_step", ctypes.c_int, [_VP]),
+    ("rikfad_check_finite", ctypes.c_int, [_VP, _VP]),
+    ("rikfad_debug_check_failures", ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_int64),
+                                                   ctypes.POINTER(ctypes.c_int)]),
+    ("rikfad_debug_fail_allocation", None, [ctypes.c_int64]),
+    ("rikfad_debug_live_allocations", ctypes.c_int64, []),
     ("rikfad_plan_query", ctypes.c_int64, [ctypes.POINTER(Shape), ctypes.c_int, ctypes.c_int,
                                            ctypes.c_int, ctypes.POINTER(ctypes.c_int64),
                                            ctypes.c_int64]),
@@ -161,13 +169,41 @@ def plan_query(shapes, grad_dtype, nblocks):
     return out[:n]
 
 
+def _check_tensor(name, t, numel, dtype):
+    """Raise ValueError unless ``t`` is a contiguous CUDA tensor of ``dtype``
+    with ``numel`` elements (the C side cannot check sizes)."""
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise ValueError("%s must be a torch tensor" % name)
+    if not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
+    if t.dtype != dtype:
+        raise ValueError("%s must be %s, not %s" % (name, dtype, t.dtype))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if t.numel() != numel:
+        raise ValueError("%s has %d elements, expected %d" % (name, t.numel(), numel))
+
+
 def step_matrix_noalloc(rows, cols, h, pending_step, alpha, mu, gamma, eps_stab, grad_dtype, x, grad,
                         p, R, C, stream=None):
     """One allocation-free step of a single matrix (``rikfad_step_matrix_noalloc``):
     the caller owns x, grad, p and the factors R, C, and remembers the
-    previous step size itself (``pending_step``)."""
+    previous step size itself (``pending_step``).  Sizes within the library's
+    limits are checked here: x, p (float32) and grad (bf16 or float32, as
+    ``grad_dtype``) must hold rows * cols elements, R rows and C cols float32
+    elements, all contiguous CUDA tensors.  Sizes beyond the limits are left
+    to the library, which refuses them."""
+    import torch
     hp = HParams(float(alpha), float(mu), float(gamma), float(eps_stab))
     gd = GRAD_BF16 if grad_dtype in ("bf16", GRAD_BF16) else GRAD_F32
+    rows, cols = int(rows), int(cols)
+    if 0 <= rows <= 65536 and 1 <= cols <= 1024:
+        gdt = torch.bfloat16 if gd == GRAD_BF16 else torch.float32
+        for name, t, n, dt in (("x", x, rows * cols, torch.float32), ("p", p, rows * cols, torch.float32),
+                               ("grad", grad, rows * cols, gdt), ("R", R, rows, torch.float32),
+                               ("C", C, cols, torch.float32)):
+            _check_tensor(name, t, n, dt)
     _check(lib().rikfad_step_matrix_noalloc(int(rows), int(cols), float(h), float(pending_step),
                                             ctypes.byref(hp), gd, _ptr(x), _ptr(grad), _ptr(p),
                                             _ptr(R), _ptr(C), _stream_ptr(stream)))
@@ -360,3 +396,26 @@ class RIKFAD:
 
     def launches_per_step(self):
         return lib().rikfad_launches_per_step(self.handle)
+
+    def check_finite(self, stream=None):
+        """Wait for the stream; raise RikfadError(ERR_NONFINITE) if a step
+        produced a non-finite factor, friction or denominator (the report is
+        then cleared)."""
+        _check(lib().rikfad_check_finite(self.handle, _stream_ptr(stream)))
+
+    def debug_check_failures(self):
+        """(failed device checks, code of the first); (-1, 0) in a library
+        built without the checks."""
+        n, code = ctypes.c_int64(), ctypes.c_int()
+        _check(lib().rikfad_debug_check_failures(self.handle, ctypes.byref(n), ctypes.byref(code)))
+        return n.value, code.value
+
+
+def debug_fail_allocation(n):
+    """Make the n-th library allocation from now on fail (n <= 0: off)."""
+    lib().rikfad_debug_fail_allocation(int(n))
+
+
+def debug_live_allocations():
+    """Allocations the library currently holds."""
+    return lib().rikfad_debug_live_allocations()

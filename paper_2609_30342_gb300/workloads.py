@@ -14,6 +14,9 @@ two-dimensional layers in GPT2-S (Section 4.4), i.e. 12 blocks x {q, k, v,
 o, fc, proj} plus the token and position embeddings.  The token embedding is
 tied to the output head and appears once.
 """
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 
 try:  # torch is only needed for the bf16 rounding of gradients
@@ -91,15 +94,43 @@ def bf16_round(a):
     return t.to(torch.bfloat16).to(torch.float32).numpy()
 
 
-def normal_list(shapes, seed, std, dtype=np.float32):
-    """One float32 array per shape, i.i.d. N(0, std^2), drawn in list order from ``seed``."""
-    rng = np.random.default_rng(seed)
-    out = []
-    for s in shapes:
-        a = rng.standard_normal(numel(s), dtype=np.float32)
-        a *= np.float32(std)
-        out.append(a.reshape(array_shape(s)).astype(dtype, copy=False))
-    return out
+_BLOCK = 1 << 22          # elements drawn from one stream
+_pool = None
+
+
+def _block_pool():
+    global _pool
+    if _pool is None:
+        _pool = ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 4))
+    return _pool
+
+
+def tensor_normal(shape, seed, std):
+    """float32 array of ``shape`` (a (rows, cols) pair), i.i.d. N(0, std^2).
+    Elements [b 2^22, (b + 1) 2^22) come from the stream [*seed, b], so the
+    blocks of a large tensor are drawn in parallel threads."""
+    n = numel(shape)
+    out = np.empty(n, np.float32)
+    base = [int(v) for v in np.atleast_1d(seed)]
+
+    def fill(b):
+        lo, hi = b * _BLOCK, min(n, (b + 1) * _BLOCK)
+        np.random.default_rng(base + [b]).standard_normal(hi - lo, dtype=np.float32, out=out[lo:hi])
+        out[lo:hi] *= np.float32(std)
+
+    nb = -(-n // _BLOCK)
+    if nb == 1:
+        fill(0)
+    elif nb > 1:
+        list(_block_pool().map(fill, range(nb)))
+    return out.reshape(array_shape(shape))
+
+
+def normal_list(shapes, seed, std):
+    """One float32 array per shape, i.i.d. N(0, std^2); tensor t draws from its
+    own stream [*seed, t], so any tensor can be drawn without the others."""
+    base = list(np.atleast_1d(seed))
+    return [tensor_normal(s, base + [t], std) for t, s in enumerate(shapes)]
 
 
 class ModelInputs:
@@ -107,22 +138,29 @@ class ModelInputs:
 
     ``X`` ~ N(0, x_std^2) float32, ``P`` = 0, and ``grads(step)`` yields
     float32 arrays ~ N(0, g_std^2), already rounded to bf16 when
-    ``grad_bf16`` (the rounded values are what both sides consume).
+    ``grad_bf16`` (the rounded values are what both sides consume).  Every
+    tensor has its own streams ([seed, 0, t] for X, [seed, 1, step, t] for
+    its gradients): ``x(t)`` and ``grad(step, t)`` draw one tensor alone.
     """
 
-    def __init__(self, shapes, seed, x_std=0.02, g_std=1e-3, grad_bf16=True):
+    def __init__(self, shapes, seed, x_std=0.02, g_std=1e-3, grad_bf16=True, draw_x=True):
         self.shapes = list(shapes)
         self.seed = int(seed)
+        self.x_std = float(x_std)
         self.g_std = float(g_std)
         self.grad_bf16 = bool(grad_bf16)
-        self.X = normal_list(self.shapes, [self.seed, 0], x_std)
-        self.P = [np.zeros(array_shape(s), np.float32) for s in self.shapes]
+        self.X = [self.x(t) for t in range(len(self.shapes))] if draw_x else None
+        self.P = [np.zeros(array_shape(s), np.float32) for s in self.shapes] if draw_x else None
+
+    def x(self, t):
+        return tensor_normal(self.shapes[t], [self.seed, 0, t], self.x_std)
+
+    def grad(self, step, t):
+        g = tensor_normal(self.shapes[t], [self.seed, 1, int(step), t], self.g_std)
+        return bf16_round(g) if self.grad_bf16 else g
 
     def grads(self, step):
-        g = normal_list(self.shapes, [self.seed, 1, int(step)], self.g_std)
-        if self.grad_bf16:
-            g = [bf16_round(a) for a in g]
-        return g
+        return [self.grad(step, t) for t in range(len(self.shapes))]
 
 
 class QuadraticProblem:

@@ -29,3 +29,18 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter):
+    # Per-element parity statistics of the GPU tests (how many elements
+    # needed the rounding bound beyond the pure relative tolerance).
+    gh = sys.modules.get("gpu_helpers")
+    if gh is not None and os.environ.get("RIKFAD_EXPECT_CHECKED"):
+        terminalreporter.write_line("checked handles: %d, failed device checks: %d"
+                                    % (len(gh.CHECKED), sum(gh.CHECKED)))
+    em = sys.modules.get("error_model")
+    if em is None or not em.STATS:
+        return
+    terminalreporter.write_sep("-", "parity: elements beyond the pure relative tolerance")
+    for line in em.summary_lines():
+        terminalreporter.write_line(line)

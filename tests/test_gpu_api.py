@@ -9,7 +9,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import rikfad, workloads
 
-from gpu_helpers import GpuRun, compare_state
+from gpu_helpers import GpuRun, Tracked
 
 pytestmark = pytest.mark.gpu
 
@@ -56,12 +56,12 @@ def test_materialize_keeps_the_trajectory():
     """Materialising between steps (P becomes canonical, pending factor
     cleared) changes only rounding: the trajectory stays on the oracle's."""
     inp, run = _run()
-    ref = oracle.ModelState(SHAPES, inp.X, inp.P)
+    ref = Tracked(run, SHAPES, inp.X, inp.P)
     for k in range(4):
         g = inp.grads(k)
         run.set_grads(g)
         run.step(0.1)
-        ref.step([a.astype(np.float64) for a in g], 0.1, HP)
+        ref.step(g, 0.1, HP, run.factors())
         if k == 1:
             assert run.opt.pending_step == pytest.approx(0.1)
             before = run.canonical_P()
@@ -70,7 +70,7 @@ def test_materialize_keeps_the_trajectory():
             after = [p.double().cpu().numpy() for p in run.p]
             for a, b in zip(before, after):
                 assert np.array_equal(a, b)   # same expression, same rounding
-    compare_state(run, ref, 1e-4, 1e-2, "after materialize ")
+    ref.check(run, 1e-4, "after materialize")
     run.close()
 
 

@@ -13,7 +13,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import workloads
 
-from gpu_helpers import GpuRun, compare, compare_state
+from gpu_helpers import GpuRun, Tracked, compare
 
 pytestmark = pytest.mark.gpu
 
@@ -51,14 +51,14 @@ def test_schedule_matches_oracle(schedule):
     inp = workloads.ModelInputs(SHAPES, seed=21, g_std=1e-2)
     run = _make(schedule, inp)
     assert run.opt.launches_per_step() == (1 if schedule == "sweep" else 2)
-    ref = oracle.ModelState(SHAPES, inp.X, inp.P)
+    ref = Tracked(run, SHAPES, inp.X, inp.P)
     hs = (0.1, 0.1, 0.05)
     for k, h in enumerate(hs):
         g = inp.grads(k)
         run.set_grads(g)
         run.step(h)
-        ref.step([a.astype(np.float64) for a in g], h, HP)
-    compare_state(run, ref, 1e-4, 1e-2, schedule + " ")
+        ref.step(g, h, HP, run.factors())
+        ref.check(run, 1e-5 if k == 0 else 1e-4, "%s step%d" % (schedule, k + 1))
     run.close()
 
 

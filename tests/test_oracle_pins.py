@@ -9,6 +9,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import workloads
 
 import pins
+from oracle import explicit
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
 
@@ -144,3 +145,37 @@ def test_energy_decreases_on_convex_quadratic(gamma):
         assert E <= E_prev * (1 + 1e-12)
         E_prev = E
     assert E_prev < 0.2 * E0
+
+
+@pytest.mark.parametrize("shape", [(1, 1), (4, 3), (7, 5), (33, 17)])
+def test_half_damped_momentum_output(shape):
+    """The oracle's optional P^(1) output (the stored form of the GPU step):
+    equal to the kick P_n - h g when the factors are zero (no friction yet,
+    so the first half-damp is the identity), and to the independent numpy
+    variant's P^(1) from non-zero factors; the main outputs are unchanged by
+    asking for it."""
+    m, n = shape
+    rng = np.random.default_rng(m * 100 + n)
+    X = rng.standard_normal((m, n))
+    P = rng.standard_normal((m, n))
+    G = rng.standard_normal((m, n))
+    hp = HParams(0.7, 0.3, 0.2, 1e-3)
+    h = 0.1
+    # zero factors: P^(1) = P^(B) exactly
+    P1 = np.empty((m, n))
+    Xa, Pa, Ra, Ca = X.copy(), P.copy(), np.zeros(m), np.zeros(n)
+    oracle.step_matrix(Xa, Pa, Ra, Ca, G, h, hp, P1=P1)
+    assert np.array_equal(P1, P - h * G)
+    Xb, Pb, Rb, Cb = X.copy(), P.copy(), np.zeros(m), np.zeros(n)
+    oracle.step_matrix(Xb, Pb, Rb, Cb, G, h, hp)
+    for a, b in ((Xa, Xb), (Pa, Pb), (Ra, Rb), (Ca, Cb)):
+        assert np.array_equal(a, b)
+    # non-zero factors: against the explicit-friction variant
+    R0 = rng.uniform(0.1, 2.0, m)
+    C0 = rng.uniform(0.1, 2.0, n)
+    Xc, Pc, Rc, Cc = X.copy(), P.copy(), R0.copy(), C0.copy()
+    oracle.step_matrix(Xc, Pc, Rc, Cc, G, h, hp, P1=P1)
+    ref = explicit.step_matrix_explicit(X, P, R0, C0, G, h, hp.alpha, hp.mu, hp.gamma, hp.eps_stab,
+                                        return_p1=True)
+    assert np.allclose(P1, ref[4], rtol=1e-13, atol=0.0)
+    assert not np.allclose(P1, P - h * G)      # the friction acted
