@@ -174,7 +174,9 @@ struct rikfad_handle_s {
     // full iKFAD with shadow R-iKFAD factors (friction diagnostics)
     bool shadow = false;
     float *d_diag_u = nullptr, *d_diag_v = nullptr, *d_diag_w = nullptr, *d_diag_wpart = nullptr;
-    double *d_diag_norms = nullptr;
+    double *d_diag_norms = nullptr, *d_diag_upart = nullptr;
+    DiagState *d_diag_state = nullptr;
+    DiagState *h_diag_state = nullptr;   // pinned
 
     // in-order ("sweep") schedule, allocated only when selected
     bool sweep = false;
@@ -307,11 +309,13 @@ void release(rikfad_handle h)
                     (void *)h->d_slot_off, (void *)h->d_fin, (void *)h->d_fac, (void *)h->d_rowpart,
                     (void *)h->d_colpart, (void *)h->d_spart, (void *)h->d_den, (void *)h->d_guard,
                     (void *)h->d_checks, (void *)h->d_diag_u, (void *)h->d_diag_v, (void *)h->d_diag_w,
-                    (void *)h->d_diag_wpart, (void *)h->d_diag_norms, (void *)h->d_units, (void *)h->d_nodes,
+                    (void *)h->d_diag_wpart, (void *)h->d_diag_norms, (void *)h->d_diag_upart,
+                    (void *)h->d_diag_state, (void *)h->d_units, (void *)h->d_nodes,
                     (void *)h->d_trees, (void *)h->d_partials, (void *)h->d_counts, (void *)h->d_fetch})
         rk_free(p);
     rk_free_host(h->h_den);
     rk_free_host(h->h_guard);
+    rk_free_host(h->h_diag_state);
     ptrtable_free(h->step_ptrs);
     ptrtable_free(h->canon_ptrs);
     for (cudaEvent_t ev : h->prof_events)
@@ -701,6 +705,13 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
         if (!rc) rc = alloc_zero(&h->d_diag_w, max_n, ws);
         if (!rc) rc = alloc_zero(&h->d_diag_wpart, max_parts * max_n, ws);
         if (!rc) rc = alloc_zero((float **)&h->d_diag_norms, 4 * ((max_m + kWarps - 1) / kWarps), ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_diag_upart, 2 * ((max_m + kWarps - 1) / kWarps), ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_diag_state, (int64_t)(sizeof(DiagState) / sizeof(float)), ws);
+        if (!rc) {
+            cudaError_t e = rk_malloc_host((void **)&h->h_diag_state, sizeof(DiagState), cudaHostAllocDefault);
+            if (e != cudaSuccess)
+                rc = alloc_fail(e, "cudaHostAlloc of the diagnostic state read-back");
+        }
     }
     if (!rc) rc = ptrtable_init(h->step_ptrs, 3 * ntensors, ws);
     if (!rc) rc = ptrtable_init(h->canon_ptrs, 2 * ntensors, ws);
@@ -1135,19 +1146,41 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     const float *xi = h->d_fac + td.xi_off;
     const float *R = h->d_fac + td.fac_off;
     const float *C = h->d_fac + td.fac_off + m;
-    // 1^T R exactly as the step kernels form it
+    // 1^T R exactly as the step kernels form it, then inv, the start vector
+    // (C normalised) and a cleared iteration state, all on the device.
     DenParams d{h->d_tensors, h->d_spart, h->d_den, h->ntensors, bounds(h)};
     rikfad_denominators_kernel<<<(h->ntensors + kWarps - 1) / kWarps, kThreads, 0, s>>>(d);
-    RK_CUDA(cudaGetLastError(), "launch rikfad_denominators_kernel");
-    float den_sum = 0.f;
-    RK_CUDA(cudaMemcpyAsync(&den_sum, h->d_den + t, sizeof(float), cudaMemcpyDeviceToHost, s), "cudaMemcpyAsync");
-    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-    const float den = den_sum + (float)h->hp.eps_stab;
-    const float inv = den == 0.f ? 0.f : 1.f / den;
+    rikfad_diag_setup_kernel<<<1, kDiagFinThreads, 0, s>>>(h->d_den + t, (float)h->hp.eps_stab, C, n,
+                                                           h->d_diag_v, h->d_diag_state);
     // ||xi||^2 and ||xi - xi~||^2
     const int nb_rows = (int)((m + kWarps - 1) / kWarps);
-    rikfad_diag_norms_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, R, C, inv, h->d_diag_norms);
-    RK_CUDA(cudaGetLastError(), "launch rikfad_diag_norms_kernel");
+    rikfad_diag_norms_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, R, C, h->d_diag_state, h->d_diag_norms);
+    RK_CUDA(cudaGetLastError(), "launch diagnostic set-up kernels");
+    // sigma_1 by power iteration on xi^T xi, starting from C (the shadow
+    // column factor, close to the top right singular vector).  Iterations
+    // are enqueued in batches; after convergence the remaining kernels of a
+    // batch return at once.  One small read-back per batch.
+    const int nb_t = (int)((m + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
+    constexpr int kBatch = 8;
+    int enqueued = 0;
+    DiagState &st = *h->h_diag_state;
+    for (;;) {
+        for (int b = 0; b < kBatch && enqueued < max_iters; ++b, ++enqueued) {
+            rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, h->d_diag_v, h->d_diag_u,
+                                                                   h->d_diag_upart, h->d_diag_state);
+            rikfad_diag_matvec_t_kernel<<<nb_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
+                                                                  h->d_diag_state);
+            rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, s>>>(h->d_diag_wpart, nb_t, n, h->d_diag_upart,
+                                                                    nb_rows, h->d_diag_w, h->d_diag_v,
+                                                                    h->d_diag_state, tol, max_iters);
+        }
+        RK_CUDA(cudaGetLastError(), "launch diagnostic kernels");
+        RK_CUDA(cudaMemcpyAsync(h->h_diag_state, h->d_diag_state, sizeof(DiagState), cudaMemcpyDeviceToHost, s),
+                "cudaMemcpyAsync diagnostic state");
+        RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+        if (st.done || enqueued >= max_iters)
+            break;
+    }
     std::vector<double> parts(2 * (size_t)nb_rows);
     RK_CUDA(cudaMemcpyAsync(parts.data(), h->d_diag_norms, sizeof(double) * parts.size(), cudaMemcpyDeviceToHost, s),
             "cudaMemcpyAsync");
@@ -1157,48 +1190,8 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
         f2 += parts[2 * b];
         e2 += parts[2 * b + 1];
     }
-    // sigma_1 by power iteration on xi^T xi, starting from C (the shadow
-    // column factor, close to the top right singular vector).
-    std::vector<float> v(n), hw(n), hu(m);
-    RK_CUDA(cudaMemcpyAsync(v.data(), C, sizeof(float) * n, cudaMemcpyDeviceToHost, s), "cudaMemcpyAsync");
-    RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-    double vn = 0.0;
-    for (float x : v)
-        vn += (double)x * x;
-    vn = std::sqrt(vn);
-    for (int64_t j = 0; j < n; ++j)
-        v[j] = vn > 0 ? (float)(v[j] / vn) : (float)(1.0 / std::sqrt((double)n));
-    const int nb_t = (int)((m + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
-    double sigma2 = 0.0;
-    int it = 0;
-    for (it = 1; it <= max_iters; ++it) {
-        RK_CUDA(cudaMemcpyAsync(h->d_diag_v, v.data(), sizeof(float) * n, cudaMemcpyHostToDevice, s),
-                "cudaMemcpyAsync");
-        rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, h->d_diag_v, h->d_diag_u);
-        rikfad_diag_matvec_t_kernel<<<nb_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart);
-        rikfad_diag_colsum_kernel<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
-            h->d_diag_wpart, nb_t, n, h->d_diag_w);
-        RK_CUDA(cudaGetLastError(), "launch diagnostic kernels");
-        RK_CUDA(cudaMemcpyAsync(hu.data(), h->d_diag_u, sizeof(float) * m, cudaMemcpyDeviceToHost, s),
-                "cudaMemcpyAsync");
-        RK_CUDA(cudaMemcpyAsync(hw.data(), h->d_diag_w, sizeof(float) * n, cudaMemcpyDeviceToHost, s),
-                "cudaMemcpyAsync");
-        RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-        double u2 = 0.0, w2 = 0.0;
-        for (float x : hu)
-            u2 += (double)x * x;
-        for (float x : hw)
-            w2 += (double)x * x;
-        const double prev = sigma2;
-        sigma2 = u2;                           // Rayleigh quotient of xi^T xi at unit v
-        if (w2 == 0.0)
-            break;
-        const double wn = std::sqrt(w2);
-        for (int64_t j = 0; j < n; ++j)
-            v[j] = (float)(hw[j] / wn);
-        if (it > 1 && std::fabs(sigma2 - prev) <= tol * sigma2)
-            break;
-    }
+    const double sigma2 = st.sigma2;
+    const int it = st.it;
     const double sigma1 = std::sqrt(sigma2);
     if (f2 > 0.0) {
         out[0] = std::sqrt(e2 / f2);                                    // ||xi - xi~|| / ||xi||

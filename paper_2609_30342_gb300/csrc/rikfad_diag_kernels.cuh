@@ -6,13 +6,28 @@
 // sigma_1^2 (the comparison of the paper's Section 4.4).  sigma_1 comes from
 // power iteration on xi^T xi: two matrix-vector passes over xi per iteration
 // (HBM-bound GEMVs; there is no dense contraction to put on tensor cores).
-// Every reduction runs in a fixed order.
+// The iteration runs on the device: a one-block kernel normalises the
+// iterate, forms the Rayleigh quotient and tests convergence, and every
+// kernel of the loop returns at once after convergence, so the host enqueues
+// iterations in batches and reads one small state record per batch.  Every
+// reduction runs in a fixed order.
 #pragma once
 #include "rikfad_kernels.cuh"
 
 namespace rikfad {
 
 constexpr int kDiagRowsPerBlock = 256;   // rows per block of the transposed product
+constexpr int kDiagFinThreads = 1024;    // threads of the one-block kernels
+
+// State of one power iteration, in device memory (read back by the host).
+struct DiagState {
+    double sigma2;     // Rayleigh quotient ||xi v||^2 of the current unit iterate
+    double w2;         // ||xi^T xi v||^2
+    int32_t it;        // iterations done
+    int32_t done;      // converged, or max_iters reached, or xi^T xi v = 0
+    float inv;         // 1 / (1^T R + eps_stab) of the shadow factors (0 if zero)
+    int32_t pad_;
+};
 
 __device__ __forceinline__ double warp_sum_f64(double v)
 {
@@ -22,15 +37,58 @@ __device__ __forceinline__ double warp_sum_f64(double v)
     return v;
 }
 
+// Block-wide sum of one double per thread, threads in a fixed tree order;
+// the result is returned to every thread.
+template <int NT>
+__device__ __forceinline__ double block_sum_f64(double v, double *scratch)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_sum_f64(v);
+    __syncthreads();
+    if (lane == 0)
+        scratch[warp] = v;
+    __syncthreads();
+    double t = 0.0;
+#pragma unroll
+    for (int k = 0; k < NT / 32; ++k)
+        t += scratch[k];
+    return t;
+}
+
+// Start of a diagnostic: inv from 1^T R (den, as the step kernels form it),
+// the unit start vector v = C / ||C|| (1/sqrt(n) per entry if C = 0), and a
+// cleared state.  One block.
+__global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_setup_kernel(const float *den, float eps,
+                                                                           const float *C, int64_t n,
+                                                                           float *v, DiagState *st)
+{
+    __shared__ double scratch[kDiagFinThreads / 32];
+    double a = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
+        a += (double)C[j] * (double)C[j];
+    const double cn = sqrt(block_sum_f64<kDiagFinThreads>(a, scratch));
+    for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
+        v[j] = cn > 0.0 ? (float)((double)C[j] / cn) : (float)(1.0 / sqrt((double)n));
+    if (threadIdx.x == 0) {
+        const float d = *den + eps;
+        st->inv = d == 0.f ? 0.f : 1.f / d;
+        st->sigma2 = 0.0;
+        st->w2 = 0.0;
+        st->it = 0;
+        st->done = 0;
+    }
+}
+
 // Per block of 8 rows (one per warp): sum of xi^2 and of (xi - xi~)^2 in
 // float64, written to part[2 * block] and part[2 * block + 1].
 __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float *xi, int64_t m, int64_t n,
                                                                      const float *R, const float *C,
-                                                                     float inv, double *part)
+                                                                     const DiagState *st, double *part)
 {
     __shared__ double s1[kWarps], s2[kWarps];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t row = (int64_t)blockIdx.x * kWarps + warp;
+    const float inv = st->inv;
     double a1 = 0.0, a2 = 0.0;
     if (row < m) {
         const float rhat = R[row] * inv;
@@ -59,27 +117,44 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float
     }
 }
 
-// u = xi v, one warp per row.
+// u = xi v, one warp per row, and per block of 8 rows the sum of u_i^2 in
+// float64 (upart[block]).  Returns at once once the iteration is done.
 __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_kernel(const float *xi, int64_t m, int64_t n,
-                                                                      const float *v, float *u)
+                                                                      const float *v, float *u, double *upart,
+                                                                      const DiagState *st)
 {
+    __shared__ double su[kWarps];
+    if (st->done)
+        return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t row = (int64_t)blockIdx.x * kWarps + warp;
-    if (row >= m)
-        return;
     float acc = 0.f;
-    for (int64_t j = lane; j < n; j += 32)
-        acc = fmaf(xi[row * n + j], v[j], acc);
-    acc = warp_sum(acc);
+    if (row < m) {
+        for (int64_t j = lane; j < n; j += 32)
+            acc = fmaf(xi[row * n + j], v[j], acc);
+        acc = warp_sum(acc);
+        if (lane == 0)
+            u[row] = acc;
+    }
     if (lane == 0)
-        u[row] = acc;
+        su[warp] = row < m ? (double)acc * (double)acc : 0.0;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int k = 0; k < kWarps; ++k)
+            t += su[k];
+        upart[blockIdx.x] = t;
+    }
 }
 
 // wpart[b][j] = sum over the rows of block b of xi_ij u_i (one thread per
-// column, rows in order).
+// column, rows in order).  Returns at once once the iteration is done.
 __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_t_kernel(const float *xi, int64_t m, int64_t n,
-                                                                        const float *u, float *wpart)
+                                                                        const float *u, float *wpart,
+                                                                        const DiagState *st)
 {
+    if (st->done)
+        return;
     const int64_t r0 = (int64_t)blockIdx.x * kDiagRowsPerBlock;
     const int64_t r1 = r0 + kDiagRowsPerBlock < m ? r0 + kDiagRowsPerBlock : m;
     for (int64_t j = threadIdx.x; j < n; j += kThreads) {
@@ -90,17 +165,46 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_t_kernel(const fl
     }
 }
 
-// w[j] = sum over blocks of wpart[b][j], blocks in order.
-__global__ void __launch_bounds__(kThreads) rikfad_diag_colsum_kernel(const float *wpart, int nb, int64_t n,
-                                                                      float *w)
+// End of one power iteration, one block: w_j = sum over blocks of
+// wpart[b][j] (blocks in order), sigma^2 = ||u||^2 (the Rayleigh quotient
+// of xi^T xi at the unit v), the next iterate v = w / ||w||, and the
+// convergence test |sigma^2 - previous| <= tol sigma^2 (from the second
+// iteration on); done after max_iters iterations or when w = 0.  w is kept
+// in w_scratch between the two passes over the columns.
+__global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
+    const float *wpart, int nb, int64_t n, const double *upart, int nbu, float *w_scratch, float *v,
+    DiagState *st, double tol, int max_iters)
 {
-    const int64_t j = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-    if (j >= n)
+    __shared__ double scratch[kDiagFinThreads / 32];
+    if (st->done)
         return;
-    float acc = 0.f;
-    for (int b = 0; b < nb; ++b)
-        acc += wpart[(int64_t)b * n + j];
-    w[j] = acc;
+    double a = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads) {
+        float acc = 0.f;
+        for (int b = 0; b < nb; ++b)
+            acc += wpart[(int64_t)b * n + j];
+        w_scratch[j] = acc;
+        a += (double)acc * (double)acc;
+    }
+    const double w2 = block_sum_f64<kDiagFinThreads>(a, scratch);
+    double c = 0.0;
+    for (int b = threadIdx.x; b < nbu; b += kDiagFinThreads)
+        c += upart[b];
+    const double u2 = block_sum_f64<kDiagFinThreads>(c, scratch);
+    if (w2 > 0.0) {
+        const double wn = sqrt(w2);
+        for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
+            v[j] = (float)((double)w_scratch[j] / wn);
+    }
+    if (threadIdx.x == 0) {
+        const double prev = st->sigma2;
+        const int it = st->it + 1;
+        st->it = it;
+        st->sigma2 = u2;
+        st->w2 = w2;
+        if (w2 == 0.0 || it >= max_iters || (it > 1 && fabs(u2 - prev) <= tol * u2))
+            st->done = 1;
+    }
 }
 
 }  // namespace rikfad
