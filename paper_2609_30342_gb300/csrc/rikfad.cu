@@ -698,7 +698,8 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
             if (td.cols > 0) {
                 max_m = std::max(max_m, td.rows);
                 max_n = std::max(max_n, td.cols);
-                max_parts = std::max<int64_t>(max_parts, (td.rows + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
+                max_parts = std::max<int64_t>(max_parts, (td.rows + diag_rows_per_group(td.rows) - 1) /
+                                                             diag_rows_per_group(td.rows));
             }
         rc = alloc_zero(&h->d_diag_u, max_m, ws);
         if (!rc) rc = alloc_zero(&h->d_diag_v, max_n, ws);
@@ -1160,7 +1161,8 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     // column factor, close to the top right singular vector).  Iterations
     // are enqueued in batches; after convergence the remaining kernels of a
     // batch return at once.  One small read-back per batch.
-    const int nb_t = (int)((m + kDiagRowsPerBlock - 1) / kDiagRowsPerBlock);
+    const int nb_t = (int)((m + diag_rows_per_group(m) - 1) / diag_rows_per_group(m));
+    const dim3 grid_t((unsigned)nb_t, (unsigned)((n + kThreads - 1) / kThreads));
     constexpr int kBatch = 8;
     int enqueued = 0;
     DiagState &st = *h->h_diag_state;
@@ -1168,8 +1170,8 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
         for (int b = 0; b < kBatch && enqueued < max_iters; ++b, ++enqueued) {
             rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, h->d_diag_v, h->d_diag_u,
                                                                    h->d_diag_upart, h->d_diag_state);
-            rikfad_diag_matvec_t_kernel<<<nb_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
-                                                                  h->d_diag_state);
+            rikfad_diag_matvec_t_kernel<<<grid_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
+                                                                    h->d_diag_state);
             rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, s>>>(h->d_diag_wpart, nb_t, n, h->d_diag_upart,
                                                                     nb_rows, h->d_diag_w, h->d_diag_v,
                                                                     h->d_diag_state, tol, max_iters);

@@ -16,8 +16,17 @@
 
 namespace rikfad {
 
-constexpr int kDiagRowsPerBlock = 256;   // rows per block of the transposed product
 constexpr int kDiagFinThreads = 1024;    // threads of the one-block kernels
+constexpr int kDiagMaxRowGroups = 64;    // row groups of the transposed product (partials per column)
+
+// Rows per block of the transposed product: at least 32, and few enough
+// row groups (at most kDiagMaxRowGroups) that the one-block finish sums
+// a short list of partials per column.
+inline __host__ __device__ int64_t diag_rows_per_group(int64_t m)
+{
+    const int64_t r = (m + kDiagMaxRowGroups - 1) / kDiagMaxRowGroups;
+    return r < 32 ? 32 : r;
+}
 
 // State of one power iteration, in device memory (read back by the host).
 struct DiagState {
@@ -147,22 +156,25 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_kernel(const floa
     }
 }
 
-// wpart[b][j] = sum over the rows of block b of xi_ij u_i (one thread per
-// column, rows in order).  Returns at once once the iteration is done.
+// wpart[g][j] = sum over the rows of row group g (blockIdx.x) of xi_ij u_i,
+// for the kThreads columns of tile blockIdx.y (one thread per column, rows
+// in order).  Returns at once once the iteration is done.
 __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_t_kernel(const float *xi, int64_t m, int64_t n,
                                                                         const float *u, float *wpart,
                                                                         const DiagState *st)
 {
     if (st->done)
         return;
-    const int64_t r0 = (int64_t)blockIdx.x * kDiagRowsPerBlock;
-    const int64_t r1 = r0 + kDiagRowsPerBlock < m ? r0 + kDiagRowsPerBlock : m;
-    for (int64_t j = threadIdx.x; j < n; j += kThreads) {
-        float acc = 0.f;
-        for (int64_t i = r0; i < r1; ++i)
-            acc = fmaf(xi[i * n + j], u[i], acc);
-        wpart[(int64_t)blockIdx.x * n + j] = acc;
-    }
+    const int64_t rpg = diag_rows_per_group(m);
+    const int64_t r0 = (int64_t)blockIdx.x * rpg;
+    const int64_t r1 = r0 + rpg < m ? r0 + rpg : m;
+    const int64_t j = (int64_t)blockIdx.y * kThreads + threadIdx.x;
+    if (j >= n)
+        return;
+    float acc = 0.f;
+    for (int64_t i = r0; i < r1; ++i)
+        acc = fmaf(xi[i * n + j], u[i], acc);
+    wpart[(int64_t)blockIdx.x * n + j] = acc;
 }
 
 // End of one power iteration, one block: w_j = sum over blocks of

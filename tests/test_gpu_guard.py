@@ -4,10 +4,8 @@ as RIKFAD_ERR_NONFINITE naming its tensor; a clean run never reports; the
 report blocks further steps until it is cleared, and a restored state steps
 again.  The division of Eq. xi_def by 1^T R + eps_stab makes one non-finite
 element poison its whole matrix, which is why the guard exists."""
-import ctypes
 import os
 
-import numpy as np
 import pytest
 import torch
 
