@@ -314,7 +314,7 @@ RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, i
  * service that allows no cudaMalloc after start-up because the call can
  * synchronise the device and stall all its streams.  This call allocates
  * nothing: the caller owns every input and output, and the partial sums live
- * in a fixed 4.45 MB array compiled into the library, which every GPU that
+ * in a fixed 1.51 MB array compiled into the library, which every GPU that
  * loads the library keeps until the process exits.
  *
  * It performs one rikfad_step on a single matrix in the same stored form:
@@ -332,11 +332,13 @@ RIKFAD_API int64_t rikfad_plan_query(const rikfad_shape *shapes, int ntensors, i
  *                 (start them at zero)
  * The first call on each device looks up the array's device address (and
  * may load the library's device code onto that GPU); make that first call
- * before any stream capture.  Every call clears the array's counter before
- * its launch and rewrites the partial sums, so calls in sequence are
- * independent.  All calls share the one array: calls whose work overlaps on
- * the GPU (unordered streams) race and give wrong results.  Errors as for
- * rikfad_step, reported through rikfad_last_error.
+ * before any stream capture.  A call enqueues three kernels on `stream` and
+ * writes every partial sum before it reads it, so nothing in the array needs
+ * to start at zero and calls in sequence are independent.  All calls share
+ * the one array: calls whose work overlaps on the GPU (unordered streams)
+ * race and give wrong results.  This call has no non-finite report (it has
+ * no handle to keep one).  Errors as for rikfad_step, reported through
+ * rikfad_last_error.
  */
 RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols, double step,
                                           double pending_step, const rikfad_hparams *hp,

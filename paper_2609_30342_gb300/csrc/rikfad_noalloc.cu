@@ -12,11 +12,12 @@
 // library image itself: every GPU that loads the library holds it until the
 // process exits.
 //
-// All calls share that one array and it keeps the last call's contents.  The
-// block counter that must start at zero is cleared by every call before its
-// launch; the partial sums are fully rewritten each call.  Two calls whose
-// kernels overlap on the GPU (different streams, no ordering) race on the
-// array and produce wrong results.
+// All calls share that one array and it keeps the last call's contents.  A
+// call needs nothing in it to start at zero: it writes every partial sum it
+// later reads (the partial sums of R, the row sums, the column partials)
+// before reading them, in three launches ordered on the caller's stream.  Two
+// calls whose kernels overlap on the GPU (different streams, no ordering)
+// race on the array and produce wrong results.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -32,13 +33,16 @@ namespace {
 
 constexpr int64_t kNaMaxRows = 65536;            // largest matrix: 65536 x 1024
 constexpr int64_t kNaMaxCols = kPanelMax;        // one column panel
-constexpr int kNaMaxBlocks = 128;
-constexpr int64_t kNaCtlFloats = 64;             // word 0: finished-block counter
-constexpr int64_t kNaScratchFloats = kNaCtlFloats + kNaMaxRows + (int64_t)kNaMaxBlocks * kNaMaxCols;
+constexpr int kNaMaxBlocks = 304;                // step blocks: 2 per SM of a GB300
+constexpr int kNaRowGroup = 1024;                // rows per partial sum of R
+constexpr int64_t kNaRsumFloats = kNaMaxRows / kNaRowGroup;     // 64
+constexpr int kNaColsPerItem = 32;               // columns per block of the column finalise
+constexpr int64_t kNaScratchFloats = kNaRsumFloats + kNaMaxRows + (int64_t)kNaMaxBlocks * kNaMaxCols;
 
 }  // namespace
 
-// 4.45 MB of scratch: counter | row sums (rows) | column partials (blocks x cols).
+// 1.51 MB of scratch: partial sums of R (64) | row sums (rows) | column
+// partials (blocks x cols).
 static __device__ __align__(256) float g_noalloc_scratch[kNaScratchFloats];
 
 namespace rikfad {
@@ -60,31 +64,51 @@ struct NoAllocParams {
     float h, ex_cur, ex_prev, damp_prev, decay, gain, eps;
 };
 
-// One launch does the whole step: every block streams its row range with the
-// same per-row code as the multi-tensor kernel, writes its column partial
-// sums, and the block that finishes last folds all partials into R and C.
+// Partial sums of R over groups of kNaRowGroup rows, in a fixed order.
+__global__ void __launch_bounds__(kThreads) rikfad_noalloc_rsum_kernel(const float *R, int64_t rows,
+                                                                       float *rsum)
+{
+    __shared__ float wsum[kWarps];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t r0 = (int64_t)blockIdx.x * kNaRowGroup;
+    float v = 0.f;
+    for (int64_t i = r0 + tid; i < rows && i < r0 + kNaRowGroup; i += kThreads)
+        v += R[i];
+    v = warp_sum(v);
+    if (lane == 0)
+        wsum[warp] = v;
+    __syncthreads();
+    if (tid == 0) {
+        float t = 0.f;
+        for (int k = 0; k < kWarps; ++k)
+            t += wsum[k];
+        rsum[blockIdx.x] = t;
+    }
+}
+
+// The streaming pass: every block takes a contiguous range of rows with the
+// same per-row code as the multi-tensor kernel and writes its column partial
+// sums; the row sums go to the scratch too.
 template <typename GT, bool REUSE>
-__global__ void __launch_bounds__(kThreads) rikfad_noalloc_step_kernel(NoAllocParams na, float *scratch)
+__global__ void __launch_bounds__(kThreads, RIKFAD_STEP_MIN_BLOCKS)
+    rikfad_noalloc_step_kernel(NoAllocParams na, float *scratch)
 {
     __shared__ __align__(16) float Cs[kPanelMax];
     __shared__ __align__(16) float red[kWarps * kPanelMax];
     __shared__ void *ptrs[3];
-    __shared__ float wsum[kWarps];
-    __shared__ int is_last;
-    unsigned *counter = reinterpret_cast<unsigned *>(scratch);
-    float *rowsum = scratch + kNaCtlFloats;
-    float *colpart = scratch + kNaCtlFloats + kNaMaxRows;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const float *rsum = scratch;
+    float *rowsum = scratch + kNaRsumFloats;
+    float *colpart = scratch + kNaRsumFloats + kNaMaxRows;
+    const int tid = threadIdx.x, lane = tid & 31;
     const int b = blockIdx.x;
     const int w = (int)na.cols;
 
-    // 1^T R, summed in the same fixed order by every block.
+    // 1^T R from the partial sums, in the same fixed order in every warp.
+    const int nrs = (int)((na.rows + kNaRowGroup - 1) / kNaRowGroup);
     float v = 0.f;
-    for (int64_t i = tid; i < na.rows; i += kThreads)
-        v += na.R[i];
-    v = warp_sum(v);
-    if (lane == 0)
-        wsum[warp] = v;
+    for (int k = lane; k < nrs; k += 32)
+        v += rsum[k];
+    const float inv = inv_denominator(warp_sum(v), na.eps);
     for (int c = tid; c < w; c += kThreads)
         Cs[c] = na.C[c];
     for (int i = tid; i < kWarps * kPanelMax; i += kThreads)
@@ -95,11 +119,6 @@ __global__ void __launch_bounds__(kThreads) rikfad_noalloc_step_kernel(NoAllocPa
         ptrs[2] = na.p;
     }
     __syncthreads();
-    float s = 0.f;
-#pragma unroll
-    for (int k = 0; k < kWarps; ++k)
-        s += wsum[k];
-    const float inv = inv_denominator(s, na.eps);
 
     StepParams a{};
     a.xptr = reinterpret_cast<float *const *>(&ptrs[0]);
@@ -139,26 +158,40 @@ __global__ void __launch_bounds__(kThreads) rikfad_noalloc_step_kernel(NoAllocPa
             t += red[k * kPanelMax + c];
         colpart[(int64_t)b * w + c] = t;
     }
+}
 
-    // The last block to get here applies the factor update.
-    __threadfence();
-    __syncthreads();
-    if (tid == 0)
-        is_last = atomicAdd(counter, 1u) == (unsigned)(na.nblocks - 1);
-    __syncthreads();
-    if (!is_last)
+// The factor filter: blocks [0, nrow) update kThreads rows of R each from the
+// row sums; the others update kNaColsPerItem columns of C each, the 8 warps
+// adding every 8th block's partial and then the warp sums in order.
+__global__ void __launch_bounds__(kThreads) rikfad_noalloc_finalize_kernel(NoAllocParams na,
+                                                                           const float *scratch, int nrow)
+{
+    __shared__ float csum[kWarps][32];
+    const float *rowsum = scratch + kNaRsumFloats;
+    const float *colpart = scratch + kNaRsumFloats + kNaMaxRows;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if ((int)blockIdx.x < nrow) {
+        const int64_t i = (int64_t)blockIdx.x * kThreads + tid;
+        if (i < na.rows)
+            na.R[i] = fmaf(na.gain, rowsum[i], na.decay * na.R[i]);
         return;
-    __threadfence();
-    for (int64_t i = tid; i < na.rows; i += kThreads)
-        na.R[i] = fmaf(na.gain, __ldcg(rowsum + i), na.decay * na.R[i]);
-    for (int c = tid; c < w; c += kThreads) {
+    }
+    const int64_t c = (int64_t)(blockIdx.x - nrow) * kNaColsPerItem + lane;
+    float acc = 0.f;
+    if (c < na.cols) {
+#pragma unroll 4
+        for (int k = warp; k < na.nblocks; k += kWarps)
+            acc += colpart[(int64_t)k * na.cols + c];
+    }
+    csum[warp][lane] = acc;
+    __syncthreads();
+    if (warp == 0 && c < na.cols) {
         float t = 0.f;
-        for (int k = 0; k < na.nblocks; ++k)
-            t += __ldcg(colpart + (int64_t)k * w + c);
+#pragma unroll
+        for (int k = 0; k < kWarps; ++k)
+            t += csum[k][lane];
         na.C[c] = fmaf(na.gain, t, na.decay * na.C[c]);
     }
-    if (tid == 0)
-        *counter = 0u;
 }
 
 // Device address of the scratch array, looked up once per device.
@@ -225,9 +258,6 @@ extern "C" RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols,
     if (rc)
         return rc;
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e = cudaMemsetAsync(scratch, 0, sizeof(float) * kNaCtlFloats, s);
-    if (e != cudaSuccess)
-        return na_fail(RIKFAD_ERR_CUDA, cudaGetErrorString(e));
 
     NoAllocParams na{};
     na.rows = rows;
@@ -247,6 +277,11 @@ extern "C" RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols,
     na.gain = std::isinf(hp->mu) ? 0.f : (float)(-std::expm1(-hp->alpha * step) / (hp->mu * hp->alpha));
     na.eps = (float)hp->eps_stab;
     const bool reuse = step == pending_step;
+    // Three launches on the caller's stream: partial sums of R, the
+    // streaming pass, the factor filter.
+    const int nrs = (int)((rows + kNaRowGroup - 1) / kNaRowGroup);
+    if (nrs > 0)
+        rikfad_noalloc_rsum_kernel<<<nrs, kThreads, 0, s>>>(R, rows, scratch);
     if (grad_dtype == RIKFAD_GRAD_BF16) {
         if (reuse)
             rikfad_noalloc_step_kernel<__nv_bfloat16, true><<<na.nblocks, kThreads, 0, s>>>(na, scratch);
@@ -258,7 +293,10 @@ extern "C" RIKFAD_API int rikfad_step_matrix_noalloc(int64_t rows, int64_t cols,
         else
             rikfad_noalloc_step_kernel<float, false><<<na.nblocks, kThreads, 0, s>>>(na, scratch);
     }
-    e = cudaGetLastError();
+    const int nrow = (int)((rows + kThreads - 1) / kThreads);
+    const int ncol = (int)((cols + kNaColsPerItem - 1) / kNaColsPerItem);
+    rikfad_noalloc_finalize_kernel<<<nrow + ncol, kThreads, 0, s>>>(na, scratch, nrow);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess)
         return na_fail(RIKFAD_ERR_CUDA, cudaGetErrorString(e));
     return RIKFAD_OK;
