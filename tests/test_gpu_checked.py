@@ -2,8 +2,9 @@
 RIKFAD_CHECKED, verifies in every kernel each plan index, range and buffer
 offset and each pointer-table entry before using it, counting failures
 instead of trapping.  The edge-shape, degenerate-hyperparameter and
-Nano-shaped parity cases run on it in a child process (the library is
-chosen when the binding first loads it), and every handle must end with
+Nano-shaped parity cases, the C-ABI behaviour tests, full iKFAD, the shadow
+handle and the in-order schedule run on it in a child process (the library
+is chosen when the binding first loads it), and every handle must end with
 zero failed checks; the parity assertions themselves hold as on the
 ordinary build."""
 import os
@@ -24,9 +25,10 @@ def test_parity_cases_on_checked_build():
     lib = pkg_build.build(checked=True)
     env = dict(os.environ, RIKFAD_LIBRARY=lib, RIKFAD_EXPECT_CHECKED="1")
     cmd = [sys.executable, "-m", "pytest", "-x", "-q", "-m", "gpu", "-p", "no:cacheprovider",
-           os.path.join(HERE, "test_gpu_parity.py"), "-k",
-           "edge_shapes or degenerate or nano_shaped_full_model",
-           os.path.join(HERE, "test_gpu_api.py")]
+           "-k", "not test_gpu_parity or edge_shapes or degenerate or nano_shaped_full_model",
+           os.path.join(HERE, "test_gpu_parity.py"), os.path.join(HERE, "test_gpu_api.py"),
+           os.path.join(HERE, "test_gpu_ikfad.py"), os.path.join(HERE, "test_gpu_diagnostics.py"),
+           os.path.join(HERE, "test_gpu_schedules.py")]
     r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=1500)
     tail = (r.stdout + r.stderr)[-3000:]
     assert r.returncode == 0, tail
