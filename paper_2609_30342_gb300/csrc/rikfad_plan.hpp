@@ -26,6 +26,14 @@ constexpr int kFinColChunk = 32;     // columns per split column item (8 warps s
 constexpr int kFinSplitSlots = 8;    // panels with more slots than this get split column items
 constexpr int kElemGranule = 8;      // element pieces start on multiples of 8 elements
 constexpr int64_t kMinBlockBytes = 64 * 1024;   // smallest share worth a block
+// The planner balances blocks on time, not bytes alone: each row of a matrix
+// panel costs its compulsory bytes plus kRowCost bytes' worth of fixed work
+// (loading R_i, the exponent scale, the row-sum shuffle, the row-partial
+// store).  Measured on GB300, step-kernel bandwidth on single matrices of
+// width w follows w * 18 / (w * 18 + 250) to within 2% from w = 64 to 2048;
+// without the term, blocks holding narrow panels (a 1600-wide matrix's
+// 64-column tail) finish last.
+constexpr int64_t kRowCost = 256;
 
 enum PieceKind : int32_t { kMatrixRows = 0, kElements = 1 };
 enum FinKind : int32_t { kFinRows = 0, kFinCols = 1 };

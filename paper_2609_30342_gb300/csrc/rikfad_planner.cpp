@@ -18,8 +18,9 @@ struct Unit {
     int32_t tensor;
     int32_t panel;
     int64_t len;    // rows or elements
-    int64_t cost;   // bytes per row or element
+    int64_t cost;   // cost per row or element: its bytes, plus kRowCost for a matrix row
     int64_t gran;   // cut granularity
+    int64_t bytes;  // compulsory bytes per row or element
 };
 
 }  // namespace
@@ -79,7 +80,7 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
             fac += round_up(td.rows, 8);
             if (td.rows > 0)
                 units.push_back({kElements, t, -1, td.rows, vector_elem_bytes(grad_bytes),
-                                 kElemGranule});
+                                 kElemGranule, vector_elem_bytes(grad_bytes)});
         } else {
             td.vec = (td.cols % 8 == 0) ? 1 : 0;
             fac += round_up(td.rows + td.cols, 8);
@@ -125,11 +126,11 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
                 col0 += widths[k];
                 pd.nch = (int32_t)ceil_div(pd.width, kChunk);
                 pd.slot_begin = pd.slot_end = 0;
-                if (td.rows > 0)
-                    units.push_back({kMatrixRows, t, (int32_t)p.panels.size(), td.rows,
-                                     pd.width * (full_matrices ? vector_elem_bytes(grad_bytes)
-                                                               : matrix_elem_bytes(grad_bytes)),
-                                     1});
+                if (td.rows > 0) {
+                    const int64_t b = pd.width * (full_matrices ? vector_elem_bytes(grad_bytes)
+                                                                : matrix_elem_bytes(grad_bytes));
+                    units.push_back({kMatrixRows, t, (int32_t)p.panels.size(), td.rows, b + kRowCost, 1, b});
+                }
                 p.panels.push_back(pd);
             }
             td.rowpart_off = rowpart;
@@ -146,10 +147,12 @@ std::string build_plan(const rikfad_shape *shapes, int ntensors, int grad_bytes,
     p.rowpart_floats = rowpart;
     p.spart_floats = (int32_t)spart;
 
-    int64_t total = 0;
-    for (const Unit &u : units)
+    int64_t total = 0, total_bytes = 0;
+    for (const Unit &u : units) {
         total += u.len * u.cost;
-    p.total_bytes = total;
+        total_bytes += u.len * u.bytes;
+    }
+    p.total_bytes = total_bytes;
 
     // Cut the unit sequence into nblocks shares of nearly equal cost.
     p.block_piece.push_back(0);

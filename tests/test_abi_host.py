@@ -60,7 +60,12 @@ ODD = [(1, 1), (1, 7), (3, 5), (257, 129), (0, 4), (5, 0), (0, 0), (13, 0), (9, 
        (2, 3000), (4096, 8), (100, 1032)]
 
 
-def _cost(shape, gb):
+# The planner's per-row cost of a matrix panel row, in bytes (kRowCost in
+# csrc/rikfad_plan.hpp): blocks are balanced on bytes plus this per row.
+ROW_COST = 256
+
+
+def _bytes(shape, gb):
     m, n = shape
     return m * (gb + 24) if n == 0 else m * n * (gb + 16)
 
@@ -95,18 +100,22 @@ def test_plan_covers_every_element_once(shapes, nblocks, grad):
     for t, hit in enumerate(hits):
         assert np.all(hit == 1), "tensor %d covered %s times" % (t, np.unique(hit))
     assert slots == list(range(len(slots))), "slots must be consecutive in piece order"
-    # Balance: no block exceeds its fair share by more than one unit of work.
+    # Balance: no block exceeds its fair share of the planner's cost (bytes,
+    # plus ROW_COST per matrix panel row) by more than one unit of work; the
+    # bytes of all pieces add up to the compulsory bytes of the list.
     if plan.size:
-        total = sum(_cost(s, gb) for s in shapes)
+        total_bytes = sum(_bytes(s, gb) for s in shapes)
         used = int(blocks.max()) + 1
         per_block = np.zeros(used)
+        bytes_sum = 0.0
         largest_unit = 0
         for b, t, kind, col0, width, beg, end, slot in plan:
-            unit = width * (gb + 16) if kind == 0 else 8 * (gb + 24)
+            unit = width * (gb + 16) + ROW_COST if kind == 0 else 8 * (gb + 24)
             largest_unit = max(largest_unit, unit)
             per_block[b] += (end - beg) * unit / (1 if kind == 0 else 8)
-        assert abs(per_block.sum() - total) < 1e-6 * total
-        fair = total / used
+            bytes_sum += (end - beg) * (width * (gb + 16) if kind == 0 else gb + 24)
+        assert abs(bytes_sum - total_bytes) < 1e-6 * total_bytes
+        fair = per_block.sum() / used
         assert per_block.max() <= fair + 2 * largest_unit + 1, (per_block.max(), fair)
 
 
