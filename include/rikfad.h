@@ -399,7 +399,7 @@ RIKFAD_API int rikfad_quadratic_run(int64_t batch, int64_t m, int64_t n, const f
  *
  * rikfad_debug_check_failures: a library compiled with -DRIKFAD_CHECKED
  * (librikfad_checked.so, built by build(checked=True)) verifies inside every
- * kernel that follows a handle's plan (step, finalise, canonical momentum,
+ * kernel of the default schedule (step, finalise, canonical momentum,
  * denominators), before each access, that the plan's block, piece, tensor, panel,
  * slot and finalise-item indices, the row, column and element ranges, the
  * offsets into the factor, partial-sum and denominator buffers, and the
