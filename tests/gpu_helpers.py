@@ -153,7 +153,7 @@ def _nblocks():
     return 2 * torch.cuda.get_device_properties(0).multi_processor_count
 
 
-def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None, workers=None):
+def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None, workers=None, hs=None):
     """A parity run at model size, in the launch configuration the benchmark
     times: the whole list steps on the GPU (gradients ~ N(0, 1e-3^2), bf16,
     from the tensors' own streams); the tensors in ``tensors`` (default all)
@@ -161,7 +161,8 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
     steps of ``compare_at`` (rtol[k] at step k, per-element bound beyond it);
     the others keep their first gradients.  The oracle runs per tensor in
     spawned worker processes after the GPU run (``oracle_jobs.tensor_trajectory``),
-    from the GPU's saved arrays and per-step factors."""
+    from the GPU's saved arrays and per-step factors.  ``hs`` (default: h at
+    every step) gives the step size of each step."""
     import multiprocessing as mp
     import os
     import shutil
@@ -175,6 +176,8 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
     names = [nm for nm, _ in named]
     T = len(shapes)
     tensors = list(range(T)) if tensors is None else list(tensors)
+    hs = [h] * steps if hs is None else list(hs)
+    assert len(hs) == steps
     inp = workloads.ModelInputs(shapes, seed=seed, draw_x=False)
     pool_t = ThreadPoolExecutor(8)
     X0 = list(pool_t.map(inp.x, range(T)))
@@ -191,7 +194,7 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
             for t, g in gs:
                 run.g[t].copy_(torch.from_numpy(g).to(run.gdt).to(run.g[t].device))
             del gs
-            run.step(h)
+            run.step(hs[k - 1])
             torch.cuda.synchronize()
             for t in fac:
                 R, C = run.opt.get_factors(t)
@@ -217,7 +220,7 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
         for t in sorted(tensors, key=lambda t: -workloads.numel(shapes[t])):
             dr, dc = depths.get(t, (0.0, 0.0))
             jobs.append(dict(shapes=shapes, shape=shapes[t], t=t, name=names[t], seed=seed,
-                             hp=(hp.alpha, hp.mu, hp.gamma, hp.eps_stab), hs=[h] * steps, steps=steps,
+                             hp=(hp.alpha, hp.mu, hp.gamma, hp.eps_stab), hs=hs, steps=steps,
                              compare_at=sorted(compare_at), rtol=rtol, dir=d, tag=tag,
                              depth_row=dr, depth_col=dc))
         nw = workers or max(1, min(len(jobs), (os.cpu_count() or 2) - 1, 16))

@@ -128,3 +128,30 @@ def test_guard_under_sweep_schedule():
         opt.check_finite()
     assert e.value.code == rikfad.ERR_NONFINITE and "first tensor: 0" in str(e.value)
     opt.close()
+
+
+def test_guard_reports_from_graph_replay():
+    """A step captured in a CUDA graph: replays enqueue the kernels without
+    rikfad_step, so the report comes from the kernels alone.  A non-finite
+    gradient written into the captured buffer between replays is reported by
+    rikfad_check_finite after the next replay; clean replays before it are not."""
+    inp, opt, x, g, p = _setup()
+    opt.step(H, x, g, p)              # eager: pointer table uploaded, h_prev = h
+    ptrs = opt.pack(x, g, p)
+    opt.step(H, ptrs=ptrs)
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graph, stream=stream):
+            opt.step(H, ptrs=ptrs, stream=stream)
+    for _ in range(3):
+        graph.replay()
+    opt.check_finite(stream)
+    g[2].view(-1)[5] = float("inf")
+    torch.cuda.synchronize()
+    graph.replay()
+    with pytest.raises(rikfad.RikfadError) as e:
+        opt.check_finite(stream)
+    assert e.value.code == rikfad.ERR_NONFINITE and "first tensor: 2" in str(e.value)
+    opt.close()
