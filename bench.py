@@ -415,13 +415,18 @@ def run_ours(args, rank, world, local_rank):
         if args.canonical:
             opt.materialize(p_arr, stream=stream)
 
+    # NVTX ranges mark the phases (ncu --nvtx --nvtx-include "timed/" selects
+    # the timed steps); one push and pop per phase or repeat, none per step.
+    nvtx = torch.cuda.nvtx
     w0 = torch.cuda.Event(enable_timing=True)
     w1 = torch.cuda.Event(enable_timing=True)
+    nvtx.range_push("warmup")
     w0.record(stream)
     for i in range(args.warmup):
         do_step(i, ptrs)
     w1.record(stream)
     torch.cuda.synchronize(dev)
+    nvtx.range_pop()
     warm_ms = w0.elapsed_time(w1) / max(args.warmup, 1)
 
     # ---- device-timed region: inputs resident in HBM (2.24 GB > 129 MB L2).
@@ -446,11 +451,13 @@ def run_ours(args, rank, world, local_rank):
         ev1 = torch.cuda.Event(enable_timing=True)
         barrier(world)
         torch.cuda.synchronize(dev)
+        nvtx.range_push("timed")
         ev0.record(stream)
         for i in range(args.steps):
             do_step(i, ptrs)
         ev1.record(stream)
         torch.cuda.synchronize(dev)
+        nvtx.range_pop()
         barrier(world)
         rep_ms.append(max_over_ranks(ev0.elapsed_time(ev1), world, dev))
     t_win1 = time.time()
@@ -458,10 +465,12 @@ def run_ours(args, rank, world, local_rank):
     # Kernel durations: the same steps again with CUDA events around each
     # launch (events between the kernels stop them from overlapping, so this
     # pass is kept out of the headline timing above).
+    nvtx.range_push("kernel events")
     opt.profile_enable(True)
     for i in range(args.steps):
         do_step(i, ptrs)
     torch.cuda.synchronize(dev)
+    nvtx.range_pop()
     step_ms, fin_ms, nrec = opt.profile_read()
     opt.profile_enable(False)
     opt.check_finite(stream)          # the timed steps produced finite factors
@@ -484,12 +493,14 @@ def run_ours(args, rank, world, local_rank):
     ptrs_host = opt.pack(x, host_views, p)
     barrier(world)
     torch.cuda.synchronize(dev)
+    nvtx.range_push("end to end")
     t0 = time.perf_counter()
     for i in range(args.steps):
         do_step(i, ptrs_host)
         opt.read_denominators(stream)
     torch.cuda.synchronize(dev)
     e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
+    nvtx.range_pop()
     barrier(world)
     e2e = {"value": aggregate(N, e2e_s / args.steps, world) / 1e9, "unit": UNIT,
            "h2d_bytes_per_step": int(sum(v.numel() for v in host_views) * 2),
