@@ -1158,31 +1158,61 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     rikfad_diag_norms_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, R, C, h->d_diag_state, h->d_diag_norms);
     RK_CUDA(cudaGetLastError(), "launch diagnostic set-up kernels");
     // sigma_1 by power iteration on xi^T xi, starting from C (the shadow
-    // column factor, close to the top right singular vector).  Iterations
-    // are enqueued in batches; after convergence the remaining kernels of a
-    // batch return at once.  One small read-back per batch.
+    // column factor, close to the top right singular vector).  A batch of
+    // kBatch iterations (three kernels each) and the read-back of the state
+    // record are captured once into a CUDA graph, which is replayed until
+    // the iteration is done; after convergence the remaining kernels of a
+    // batch return at once.  (The iterations are small kernels: launched one
+    // by one, their launch costs dominated.)
     const int nb_t = (int)((m + diag_rows_per_group(m) - 1) / diag_rows_per_group(m));
     const dim3 grid_t((unsigned)nb_t, (unsigned)((n + kThreads - 1) / kThreads));
     constexpr int kBatch = 8;
-    int enqueued = 0;
     DiagState &st = *h->h_diag_state;
-    for (;;) {
-        for (int b = 0; b < kBatch && enqueued < max_iters; ++b, ++enqueued) {
-            rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, s>>>(xi, m, n, h->d_diag_v, h->d_diag_u,
-                                                                   h->d_diag_upart, h->d_diag_state);
-            rikfad_diag_matvec_t_kernel<<<grid_t, kThreads, 0, s>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
-                                                                    h->d_diag_state);
-            rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, s>>>(h->d_diag_wpart, nb_t, n, h->d_diag_upart,
-                                                                    nb_rows, h->d_diag_w, h->d_diag_v,
-                                                                    h->d_diag_state, tol, max_iters);
+    cudaStream_t cs = nullptr;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    auto cleanup = [&]() {
+        if (exec)
+            cudaGraphExecDestroy(exec);
+        if (graph)
+            cudaGraphDestroy(graph);
+        if (cs)
+            cudaStreamDestroy(cs);
+    };
+    cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
+    if (e == cudaSuccess)
+        e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal);
+    if (e == cudaSuccess) {
+        for (int b = 0; b < kBatch; ++b) {
+            rikfad_diag_matvec_kernel<<<nb_rows, kThreads, 0, cs>>>(xi, m, n, h->d_diag_v, h->d_diag_u,
+                                                                    h->d_diag_upart, h->d_diag_state);
+            rikfad_diag_matvec_t_kernel<<<grid_t, kThreads, 0, cs>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
+                                                                     h->d_diag_state);
+            rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, cs>>>(h->d_diag_wpart, nb_t, n, h->d_diag_upart,
+                                                                     nb_rows, h->d_diag_w, h->d_diag_v,
+                                                                     h->d_diag_state, tol, max_iters);
         }
-        RK_CUDA(cudaGetLastError(), "launch diagnostic kernels");
-        RK_CUDA(cudaMemcpyAsync(h->h_diag_state, h->d_diag_state, sizeof(DiagState), cudaMemcpyDeviceToHost, s),
-                "cudaMemcpyAsync diagnostic state");
-        RK_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-        if (st.done || enqueued >= max_iters)
+        cudaMemcpyAsync(h->h_diag_state, h->d_diag_state, sizeof(DiagState), cudaMemcpyDeviceToHost, cs);
+        e = cudaStreamEndCapture(cs, &graph);
+    }
+    if (e == cudaSuccess)
+        e = cudaGraphInstantiate(&exec, graph, 0);
+    if (e != cudaSuccess) {
+        cleanup();
+        return cuda_fail(e, "capture of the power iteration");
+    }
+    for (int enqueued = 0; enqueued < max_iters; enqueued += kBatch) {
+        e = cudaGraphLaunch(exec, s);
+        if (e == cudaSuccess)
+            e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) {
+            cleanup();
+            return cuda_fail(e, "power iteration");
+        }
+        if (st.done)
             break;
     }
+    cleanup();
     std::vector<double> parts(2 * (size_t)nb_rows);
     RK_CUDA(cudaMemcpyAsync(parts.data(), h->d_diag_norms, sizeof(double) * parts.size(), cudaMemcpyDeviceToHost, s),
             "cudaMemcpyAsync");

@@ -17,6 +17,7 @@
 namespace rikfad {
 
 constexpr int kDiagFinThreads = 1024;    // threads of the one-block kernels
+constexpr int kDiagBatch = 8;            // loads a thread issues before consuming them
 constexpr int kDiagMaxRowGroups = 64;    // row groups of the transposed product (partials per column)
 
 // Rows per block of the transposed product: at least 32, and few enough
@@ -47,7 +48,9 @@ __device__ __forceinline__ double warp_sum_f64(double v)
 }
 
 // Block-wide sum of one double per thread, threads in a fixed tree order;
-// the result is returned to every thread.
+// the result is returned to every thread.  Float64 arithmetic is slow on
+// this GPU, so only warp 0 combines the warp sums and the total is passed on
+// through shared memory (scratch holds NT / 32 + 1 doubles).
 template <int NT>
 __device__ __forceinline__ double block_sum_f64(double v, double *scratch)
 {
@@ -57,11 +60,14 @@ __device__ __forceinline__ double block_sum_f64(double v, double *scratch)
     if (lane == 0)
         scratch[warp] = v;
     __syncthreads();
-    double t = 0.0;
-#pragma unroll
-    for (int k = 0; k < NT / 32; ++k)
-        t += scratch[k];
-    return t;
+    if (warp == 0) {
+        double t = lane < NT / 32 ? scratch[lane] : 0.0;
+        t = warp_sum_f64(t);
+        if (lane == 0)
+            scratch[NT / 32] = t;
+    }
+    __syncthreads();
+    return scratch[NT / 32];
 }
 
 // Start of a diagnostic: inv from 1^T R (den, as the step kernels form it),
@@ -71,13 +77,21 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_setup_kernel(cons
                                                                            const float *C, int64_t n,
                                                                            float *v, DiagState *st)
 {
-    __shared__ double scratch[kDiagFinThreads / 32];
+    __shared__ double scratch[kDiagFinThreads / 32 + 1];
+    __shared__ double s_scale;
     double a = 0.0;
     for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
         a += (double)C[j] * (double)C[j];
-    const double cn = sqrt(block_sum_f64<kDiagFinThreads>(a, scratch));
+    const double c2 = block_sum_f64<kDiagFinThreads>(a, scratch);
+    // One float64 square root and division for the block (float64 is slow on
+    // this GPU), then a multiply per entry.
+    if (threadIdx.x == 0)
+        s_scale = c2 > 0.0 ? 1.0 / sqrt(c2) : 0.0;
+    __syncthreads();
+    const double sc = s_scale;
+    const float uniform = (float)(1.0 / sqrt((double)n));
     for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
-        v[j] = cn > 0.0 ? (float)((double)C[j] / cn) : (float)(1.0 / sqrt((double)n));
+        v[j] = sc > 0.0 ? (float)((double)C[j] * sc) : uniform;
     if (threadIdx.x == 0) {
         const float d = *den + eps;
         st->inv = d == 0.f ? 0.f : 1.f / d;
@@ -101,11 +115,21 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float
     double a1 = 0.0, a2 = 0.0;
     if (row < m) {
         const float rhat = R[row] * inv;
-        for (int64_t j = lane; j < n; j += 32) {
-            const float v = xi[row * n + j];
-            const double d = (double)v - (double)(rhat * C[j]);
-            a1 += (double)v * (double)v;
-            a2 += d * d;
+        // kDiagBatch loads in flight per lane, then the sums in element order
+        for (int64_t j0 = lane; j0 < n; j0 += 32 * kDiagBatch) {
+            float xv[kDiagBatch], cv[kDiagBatch];
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k) {
+                const int64_t j = j0 + 32 * k;
+                xv[k] = j < n ? xi[row * n + j] : 0.f;
+                cv[k] = j < n ? C[j] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k) {
+                const double d = (double)xv[k] - (double)(rhat * cv[k]);
+                a1 += (double)xv[k] * (double)xv[k];
+                a2 += d * d;
+            }
         }
     }
     a1 = warp_sum_f64(a1);
@@ -139,8 +163,18 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_kernel(const floa
     const int64_t row = (int64_t)blockIdx.x * kWarps + warp;
     float acc = 0.f;
     if (row < m) {
-        for (int64_t j = lane; j < n; j += 32)
-            acc = fmaf(xi[row * n + j], v[j], acc);
+        for (int64_t j0 = lane; j0 < n; j0 += 32 * kDiagBatch) {
+            float a[kDiagBatch], b[kDiagBatch];
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k) {
+                const int64_t j = j0 + 32 * k;
+                a[k] = j < n ? xi[row * n + j] : 0.f;
+                b[k] = j < n ? v[j] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k)
+                acc = fmaf(a[k], b[k], acc);
+        }
         acc = warp_sum(acc);
         if (lane == 0)
             u[row] = acc;
@@ -172,8 +206,18 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_t_kernel(const fl
     if (j >= n)
         return;
     float acc = 0.f;
-    for (int64_t i = r0; i < r1; ++i)
-        acc = fmaf(xi[i * n + j], u[i], acc);
+    for (int64_t i0 = r0; i0 < r1; i0 += kDiagBatch) {
+        float a[kDiagBatch], b[kDiagBatch];
+#pragma unroll
+        for (int k = 0; k < kDiagBatch; ++k) {
+            const int64_t i = i0 + k;
+            a[k] = i < r1 ? xi[i * n + j] : 0.f;
+            b[k] = i < r1 ? u[i] : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < kDiagBatch; ++k)
+            acc = fmaf(a[k], b[k], acc);
+    }
     wpart[(int64_t)blockIdx.x * n + j] = acc;
 }
 
@@ -187,14 +231,22 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
     const float *wpart, int nb, int64_t n, const double *upart, int nbu, float *w_scratch, float *v,
     DiagState *st, double tol, int max_iters)
 {
-    __shared__ double scratch[kDiagFinThreads / 32];
+    __shared__ double scratch[kDiagFinThreads / 32 + 1];
+    __shared__ double s_scale;
     if (st->done)
         return;
     double a = 0.0;
     for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads) {
         float acc = 0.f;
-        for (int b = 0; b < nb; ++b)
-            acc += wpart[(int64_t)b * n + j];
+        for (int b0 = 0; b0 < nb; b0 += kDiagBatch) {
+            float t[kDiagBatch];
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k)
+                t[k] = b0 + k < nb ? wpart[(int64_t)(b0 + k) * n + j] : 0.f;
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k)
+                acc += t[k];
+        }
         w_scratch[j] = acc;
         a += (double)acc * (double)acc;
     }
@@ -203,10 +255,13 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
     for (int b = threadIdx.x; b < nbu; b += kDiagFinThreads)
         c += upart[b];
     const double u2 = block_sum_f64<kDiagFinThreads>(c, scratch);
+    if (threadIdx.x == 0)
+        s_scale = w2 > 0.0 ? 1.0 / sqrt(w2) : 0.0;
+    __syncthreads();
     if (w2 > 0.0) {
-        const double wn = sqrt(w2);
+        const double sc = s_scale;
         for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
-            v[j] = (float)((double)w_scratch[j] / wn);
+            v[j] = (float)((double)w_scratch[j] * sc);
     }
     if (threadIdx.x == 0) {
         const double prev = st->sigma2;
