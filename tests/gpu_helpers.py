@@ -238,7 +238,7 @@ class Tracked:
     GPU's factors after every step give the deviations the bound takes for
     the exponents of the next step (the factors themselves are compared too)."""
 
-    def __init__(self, run, shapes, X, P, factors=None, depths=None):
+    def __init__(self, shapes, X, P, factors=None, depths=None):
         self.shapes = [tuple(s) for s in shapes]
         self.st = oracle.ModelState(self.shapes, X, P)
         if factors is not None:
@@ -255,7 +255,7 @@ class Tracked:
     @classmethod
     def from_gpu(cls, run, depths=None):
         """A fresh track from the GPU run's current state (bounds zero)."""
-        return cls(run, run.shapes, run.X(), run.canonical_P(), run.factors(), depths)
+        return cls(run.shapes, run.X(), run.canonical_P(), run.factors(), depths)
 
     def step(self, grads, h, hp, gpu_factors):
         st = self.st

@@ -56,7 +56,7 @@ def test_materialize_keeps_the_trajectory():
     """Materialising between steps (P becomes canonical, pending factor
     cleared) changes only rounding: the trajectory stays on the oracle's."""
     inp, run = _run()
-    ref = Tracked(run, SHAPES, inp.X, inp.P)
+    ref = Tracked(SHAPES, inp.X, inp.P)
     for k in range(4):
         g = inp.grads(k)
         run.set_grads(g)

@@ -35,7 +35,7 @@ def test_ikfad_matches_oracle(grad_bf16):
     inp = workloads.ModelInputs(SHAPES, seed=11, g_std=1e-2, grad_bf16=grad_bf16)
     run = GpuRun(SHAPES, hp, grad_bf16, inp.X, inp.P, method="ikfad")
     flat = _flat(SHAPES)
-    ref = Tracked(run, flat, [a.ravel() for a in inp.X], [a.ravel() for a in inp.P])
+    ref = Tracked(flat, [a.ravel() for a in inp.X], [a.ravel() for a in inp.P])
 
     def gpu_state():
         # the handle holds canonical momenta; every tensor is element-wise
@@ -45,7 +45,7 @@ def test_ikfad_matches_oracle(grad_bf16):
     for k, h in enumerate((0.1, 0.1, 0.05, 0.2)):
         g = inp.grads(k)
         X0, P0, F0 = gpu_state()
-        seeded = Tracked(run, flat, X0, P0, F0)
+        seeded = Tracked(flat, X0, P0, F0)
         run.set_grads(g)
         run.step(h)
         gflat = [a.ravel() for a in g]

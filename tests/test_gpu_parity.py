@@ -45,7 +45,7 @@ def test_single_matrix_every_step():
     shapes = [(256, 512)]
     dep = _depths(shapes)
     run = GpuRun(shapes, hp, False, [X0], [P0])
-    ref = Tracked(run, shapes, [X0], [P0], depths=dep)
+    ref = Tracked(shapes, [X0], [P0], depths=dep)
     for k in range(1, 11):
         seeded = Tracked.from_gpu(run, dep)
         run.set_grads([G[k - 1]])
@@ -66,7 +66,7 @@ def test_single_matrix_100_steps():
     X0, P0, G = workloads.single_matrix_inputs(256, 512, seed=0, steps=100)
     shapes = [(256, 512)]
     run = GpuRun(shapes, hp, False, [X0], [P0])
-    ref = Tracked(run, shapes, [X0], [P0], depths=_depths(shapes))
+    ref = Tracked(shapes, [X0], [P0], depths=_depths(shapes))
     for k in range(100):
         run.set_grads([G[k]])
         run.step(h)

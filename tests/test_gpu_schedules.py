@@ -51,7 +51,7 @@ def test_schedule_matches_oracle(schedule):
     inp = workloads.ModelInputs(SHAPES, seed=21, g_std=1e-2)
     run = _make(schedule, inp)
     assert run.opt.launches_per_step() == (1 if schedule == "sweep" else 2)
-    ref = Tracked(run, SHAPES, inp.X, inp.P)
+    ref = Tracked(SHAPES, inp.X, inp.P)
     hs = (0.1, 0.1, 0.05)
     for k, h in enumerate(hs):
         g = inp.grads(k)
