@@ -1162,8 +1162,7 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     // kBatch iterations (three kernels each) and the read-back of the state
     // record are captured once into a CUDA graph, which is replayed until
     // the iteration is done; after convergence the remaining kernels of a
-    // batch return at once.  (The iterations are small kernels: launched one
-    // by one, their launch costs dominated.)
+    // batch return at once.  One graph launch replaces 24 kernel launches.
     const int nb_t = (int)((m + diag_rows_per_group(m) - 1) / diag_rows_per_group(m));
     const dim3 grid_t((unsigned)nb_t, (unsigned)((n + kThreads - 1) / kThreads));
     constexpr int kBatch = 8;
