@@ -145,12 +145,15 @@ def test_guard_reports_from_graph_replay():
     with torch.cuda.stream(stream):
         with torch.cuda.graph(graph, stream=stream):
             opt.step(H, ptrs=ptrs, stream=stream)
-    for _ in range(3):
-        graph.replay()
+    # Replays go to the stream that check_finite waits on.
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            graph.replay()
     opt.check_finite(stream)
     g[2].view(-1)[5] = float("inf")
     torch.cuda.synchronize()
-    graph.replay()
+    with torch.cuda.stream(stream):
+        graph.replay()
     with pytest.raises(rikfad.RikfadError) as e:
         opt.check_finite(stream)
     assert e.value.code == rikfad.ERR_NONFINITE and "first tensor: 2" in str(e.value)
