@@ -306,6 +306,18 @@ def test_large_matrix_sweep(shape):
                  {1: 1e-5, 2: 1e-4})
 
 
+def test_large_matrix_sweep_100_steps():
+    """The sweep's square, wide and tall matrices (4096 x 4096, 4096 x 14336,
+    14336 x 4096; seed 4) stepped together for 100 steps with fresh
+    gradients every step: every element of all three against the oracle at
+    1e-4 (per-element rounding bound beyond it).  The 50304 x 4096 matrix,
+    tall like 14336 x 4096 and 3.5 times its size, is compared after one and
+    two steps only (test_large_matrix_sweep): its 100-step float64 oracle
+    alone takes about ten minutes."""
+    named = [("W%dx%d" % s, s) for s in workloads.SWEEP_SHAPES[:3]]
+    model_parity("sweep 100", named, 4, GPT2S_HP, GPT2S_H, 100, {100}, {100: 1e-4})
+
+
 def test_offsets_beyond_2_31_elements():
     """Maximum sizes: a 65536 x 40960 matrix (2,684,354,560 elements) and a
     vector of 2^31 + 8 elements, so element offsets pass 2^31 in every
