@@ -250,6 +250,18 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
  * non-finite result; the report stays until rikfad_check_finite clears it. */
 RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *stream);
 
+/* The same read-back, enqueued only: the denominators kernel and a copy of
+ * the ntensors floats into host_out are enqueued on `stream` and the call
+ * returns at once, so a training loop can read step n's values while step
+ * n + 1 runs (wait on the stream, or an event recorded after this call,
+ * before reading host_out).  host_out: host memory the caller owns, page-locked
+ * (cudaHostAlloc or cudaHostRegister) for the read-back to run asynchronously;
+ * when it is mapped into the device's address space the kernel stores there
+ * directly, otherwise a copy follows the kernel.  It must stay valid until
+ * the stream has passed this point.  Non-finite results are reported by
+ * rikfad_check_finite, not by this call. */
+RIKFAD_API int rikfad_enqueue_denominators(rikfad_handle h, float *host_out, void *stream);
+
 /*
  * Checkpoint support.  The state image is rikfad_state_image_bytes(h) bytes:
  * a 64-byte header (format tag, tensor count, pending step) followed by

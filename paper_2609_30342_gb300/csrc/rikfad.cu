@@ -986,6 +986,36 @@ RIKFAD_API int rikfad_read_denominators(rikfad_handle h, float *host_out, void *
     return nonfinite_status(h, s);
 }
 
+RIKFAD_API int rikfad_enqueue_denominators(rikfad_handle h, float *host_out, void *stream)
+{
+    int rc = check_handle(h);
+    if (rc)
+        return rc;
+    if (host_out == nullptr)
+        return fail(RIKFAD_ERR_ARG, "host_out is NULL");
+    const int T = h->ntensors;
+    if (T == 0)
+        return RIKFAD_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    // Page-locked memory mapped into the device's address space takes the
+    // kernel's stores directly, so no copy sits between this step's finalise
+    // and the next step's kernels (PDL launches chain through); other host
+    // memory gets a copy from the device buffer.
+    float *direct = nullptr;
+    if (cudaHostGetDevicePointer((void **)&direct, host_out, 0) != cudaSuccess) {
+        cudaGetLastError();     // not mapped: clear the query's error
+        direct = nullptr;
+    }
+    DenParams d{h->d_tensors, h->d_spart, direct ? direct : h->d_den, T, bounds(h)};
+    const int warps = 8;
+    RK_CUDA(launch_pdl(rikfad_denominators_kernel, (T + warps - 1) / warps, 32 * warps, s, d),
+            "launch rikfad_denominators_kernel");
+    if (!direct)
+        RK_CUDA(cudaMemcpyAsync(host_out, h->d_den, sizeof(float) * T, cudaMemcpyDeviceToHost, s),
+                "cudaMemcpyAsync denominators");
+    return RIKFAD_OK;
+}
+
 RIKFAD_API size_t rikfad_state_image_bytes(rikfad_handle h)
 {
     return h ? kImageHeader + sizeof(float) * (size_t)h->plan.fac_floats : 0;

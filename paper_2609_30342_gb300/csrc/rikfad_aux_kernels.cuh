@@ -275,8 +275,12 @@ __global__ void __launch_bounds__(kThreads) rikfad_canonical_kernel(CanonParams 
 }
 
 // 1^T R of every matrix (0 for vectors), same summation order as the kernels.
+// d.out may be page-locked host memory mapped into the device's address
+// space (the enqueued read-back writes there directly).
 __global__ void rikfad_denominators_kernel(DenParams d)
 {
+    wait_for_predecessor();
+    allow_successor_launch();
     const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
     if (t >= d.ntensors)
         return;

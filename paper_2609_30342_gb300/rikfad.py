@@ -67,6 +67,7 @@ SIGNATURES = [
     ("rikfad_get_factors", ctypes.c_int, [_VP, ctypes.c_int, _VP, _VP]),
     ("rikfad_set_factors", ctypes.c_int, [_VP, ctypes.c_int, _VP, _VP]),
     ("rikfad_read_denominators", ctypes.c_int, [_VP, _VP, _VP]),
+    ("rikfad_enqueue_denominators", ctypes.c_int, [_VP, _VP, _VP]),
     ("rikfad_get_friction", ctypes.c_int, [_VP, ctypes.c_int, _VP]),
     ("rikfad_friction_diagnostics", ctypes.c_int, [_VP, ctypes.c_int, ctypes.c_int, ctypes.c_double,
                                                    ctypes.POINTER(ctypes.c_double), _VP]),
@@ -374,6 +375,17 @@ class RIKFAD:
         out = np.zeros(max(len(self.shapes), 1), np.float32)
         _check(lib().rikfad_read_denominators(self.handle, out.ctypes.data, _stream_ptr(stream)))
         return out[:len(self.shapes)]
+
+    def enqueue_denominators(self, out, stream=None):
+        """Enqueue the read-back of the friction denominators into ``out``, a
+        page-locked float32 CPU tensor of at least len(shapes) elements;
+        the values are there once ``stream`` passes this point."""
+        import torch
+        if not (isinstance(out, torch.Tensor) and out.device.type == "cpu" and out.is_pinned() and
+                out.dtype == torch.float32 and out.is_contiguous() and out.numel() >= len(self.shapes)):
+            raise ValueError("out must be a contiguous page-locked float32 CPU tensor of at least %d "
+                             "elements" % len(self.shapes))
+        _check(lib().rikfad_enqueue_denominators(self.handle, out.data_ptr(), _stream_ptr(stream)))
 
     def state_image_bytes(self):
         return lib().rikfad_state_image_bytes(self.handle)

@@ -264,3 +264,44 @@ def test_pinned_host_gradients_read_in_place():
         assert torch.equal(a, b)
     run_d.close()
     run_h.close()
+
+
+def test_enqueued_denominators_match_the_synchronous_read():
+    """rikfad_enqueue_denominators writes, once the stream passes it, the
+    values rikfad_read_denominators returns; read back one step late (while
+    the next step runs), every step's values equal 1^T R of that step's
+    factors, and element-wise tensors read 0."""
+    inp, run = _run()
+    stream = torch.cuda.Stream()
+    bufs = [torch.zeros(len(SHAPES), dtype=torch.float32).pin_memory() for _ in range(2)]
+    events = [torch.cuda.Event() for _ in range(2)]
+    expect = []
+    with torch.cuda.stream(stream):
+        for k, h in enumerate((0.1, 0.1, 0.05, 0.05)):
+            run.set_grads(inp.grads(k))
+            run.opt.step(h, ptrs=run.ptrs, stream=stream)
+            run.opt.enqueue_denominators(bufs[k % 2], stream)
+            events[k % 2].record(stream)
+            if k > 0:
+                events[(k - 1) % 2].synchronize()
+                got = bufs[(k - 1) % 2].numpy().copy()
+                assert np.array_equal(got, expect[-1])
+            stream.synchronize()
+            sync = run.opt.read_denominators(stream)
+            F = run.factors()
+            for t, (m, n) in enumerate(SHAPES):
+                if n == 0:
+                    assert sync[t] == 0.0
+                else:
+                    assert sync[t] == pytest.approx(float(np.sum(F[t][0], dtype=np.float64)), rel=1e-5)
+            expect.append(sync)
+    events[1].synchronize()
+    assert np.array_equal(bufs[1].numpy(), expect[-1])
+    with pytest.raises(ValueError):
+        run.opt.enqueue_denominators(torch.zeros(len(SHAPES)))     # not page-locked
+    # Through the C ABI, pageable host memory takes the copy path.
+    pageable = np.full(len(SHAPES), -1.0, np.float32)
+    assert rikfad.lib().rikfad_enqueue_denominators(run.opt.handle, pageable.ctypes.data, None) == rikfad.OK
+    torch.cuda.synchronize()
+    assert np.array_equal(pageable, expect[-1])
+    run.close()
