@@ -64,7 +64,7 @@ def compare(name, gpu, ref, rtol, floor, atol=0.0):
     return {"max_rel": float(np.max(rel)), "beyond_pure": int(beyond.sum())}
 
 
-class GpuRun:
+class DeviceRun:
     """R-iKFAD on the GPU through the C ABI, with host-side inputs."""
 
     def __init__(self, shapes, hp, grad_bf16, X, P, device="cuda", method="rikfad"):
@@ -182,7 +182,7 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
     pool_t = ThreadPoolExecutor(8)
     X0 = list(pool_t.map(inp.x, range(T)))
     P0 = [np.zeros(workloads.array_shape(s), np.float32) for s in shapes]
-    run = GpuRun(shapes, hp, True, X0, P0)
+    run = DeviceRun(shapes, hp, True, X0, P0)
     del X0, P0
     d = tempfile.mkdtemp(prefix="rikfad_parity_")
     depths = summation_depths(shapes, _nblocks())
@@ -234,7 +234,7 @@ def model_parity(tag, named, seed, hp, h, steps, compare_at, rtol, tensors=None,
 
 class Tracked:
     """The oracle's state of a tensor list with the carried per-element
-    bounds, stepped in this process alongside a GpuRun (small cases).  The
+    bounds, stepped in this process alongside a DeviceRun (small cases).  The
     GPU's factors after every step give the deviations the bound takes for
     the exponents of the next step (the factors themselves are compared too)."""
 

@@ -9,7 +9,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import rikfad, workloads
 
-from gpu_helpers import GpuRun, Tracked
+from gpu_helpers import DeviceRun, Tracked
 
 pytestmark = pytest.mark.gpu
 
@@ -25,7 +25,7 @@ def built():
 
 def _run(seed=0, grad_bf16=True):
     inp = workloads.ModelInputs(SHAPES, seed=seed, g_std=1e-2, grad_bf16=grad_bf16)
-    return inp, GpuRun(SHAPES, HP, grad_bf16, inp.X, inp.P)
+    return inp, DeviceRun(SHAPES, HP, grad_bf16, inp.X, inp.P)
 
 
 def _state(run):

@@ -10,7 +10,7 @@ import oracle
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import workloads
 
-from gpu_helpers import GpuRun, compare
+from gpu_helpers import DeviceRun, compare
 
 pytestmark = pytest.mark.gpu
 
@@ -70,7 +70,7 @@ def _compare(run, ref, rtol, tag):
 @pytest.mark.parametrize("grad_bf16", [True, False])
 def test_shadow_run_matches_oracle(grad_bf16):
     inp = workloads.ModelInputs(SHAPES, seed=41, g_std=1e-2, grad_bf16=grad_bf16)
-    run = GpuRun(SHAPES, HP, grad_bf16, inp.X, inp.P, method="ikfad_shadow")
+    run = DeviceRun(SHAPES, HP, grad_bf16, inp.X, inp.P, method="ikfad_shadow")
     ref = ShadowRef(SHAPES, inp.X, inp.P)
     for k, h in enumerate((0.1, 0.1, 0.05, 0.2)):
         X, P, XI, RC = _gpu_state(run)
@@ -92,7 +92,7 @@ def test_diagnostics_match_dense_linear_algebra():
     computation (SVD for sigma_1): error, floor, stable rank, sigma_1, norm."""
     shapes = [(600, 768), (129, 257), (64, 1032), (2000, 64)]
     inp = workloads.ModelInputs(shapes, seed=42, g_std=1e-2)
-    run = GpuRun(shapes, HP, True, inp.X, inp.P, method="ikfad_shadow")
+    run = DeviceRun(shapes, HP, True, inp.X, inp.P, method="ikfad_shadow")
     for k in range(6):
         run.set_grads(inp.grads(k))
         run.step(0.1)
@@ -118,7 +118,7 @@ def test_rank1_momentum_gives_zero_construction_error_on_gpu():
     rng = np.random.default_rng(43)
     m, n = 256, 512
     a, b = rng.standard_normal(m).astype(np.float32), rng.standard_normal(n).astype(np.float32)
-    run = GpuRun([(m, n)], hp, False, [np.zeros((m, n), np.float32)], [np.outer(a, b)],
+    run = DeviceRun([(m, n)], hp, False, [np.zeros((m, n), np.float32)], [np.outer(a, b)],
                  method="ikfad_shadow")
     run.set_grads([np.zeros((m, n), np.float32)])
     run.step(0.3)

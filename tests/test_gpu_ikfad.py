@@ -7,7 +7,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import workloads
 
-from gpu_helpers import GpuRun, Tracked, compare
+from gpu_helpers import DeviceRun, Tracked, compare
 
 pytestmark = pytest.mark.gpu
 
@@ -33,7 +33,7 @@ def test_ikfad_matches_oracle(grad_bf16):
     bound beyond the relative tolerance."""
     hp = HParams(alpha=0.3, mu=1e-3, gamma=0.1, eps_stab=1e-8)
     inp = workloads.ModelInputs(SHAPES, seed=11, g_std=1e-2, grad_bf16=grad_bf16)
-    run = GpuRun(SHAPES, hp, grad_bf16, inp.X, inp.P, method="ikfad")
+    run = DeviceRun(SHAPES, hp, grad_bf16, inp.X, inp.P, method="ikfad")
     flat = _flat(SHAPES)
     ref = Tracked(flat, [a.ravel() for a in inp.X], [a.ravel() for a in inp.P])
 
@@ -70,8 +70,8 @@ def test_rank1_momentum_gives_identical_friction(m, n):
     b = rng.standard_normal(n).astype(np.float32)
     X = rng.standard_normal((m, n)).astype(np.float32)
     P = np.outer(a, b).astype(np.float32)
-    r1 = GpuRun([(m, n)], hp, False, [X], [P], method="rikfad")
-    fk = GpuRun([(m, n)], hp, False, [X], [P], method="ikfad")
+    r1 = DeviceRun([(m, n)], hp, False, [X], [P], method="rikfad")
+    fk = DeviceRun([(m, n)], hp, False, [X], [P], method="ikfad")
     for r in (r1, fk):
         r.set_grads([np.zeros((m, n), np.float32)])
         r.step(0.3)

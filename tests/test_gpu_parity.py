@@ -12,7 +12,7 @@ from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import rikfad, workloads
 
 import oracle_jobs
-from gpu_helpers import GpuRun, Tracked, compare, model_parity, summation_depths
+from gpu_helpers import DeviceRun, Tracked, compare, model_parity, summation_depths
 
 pytestmark = pytest.mark.gpu
 
@@ -44,7 +44,7 @@ def test_single_matrix_every_step():
     X0, P0, G = workloads.single_matrix_inputs(256, 512, seed=0, steps=10)
     shapes = [(256, 512)]
     dep = _depths(shapes)
-    run = GpuRun(shapes, hp, False, [X0], [P0])
+    run = DeviceRun(shapes, hp, False, [X0], [P0])
     ref = Tracked(shapes, [X0], [P0], depths=dep)
     for k in range(1, 11):
         seeded = Tracked.from_gpu(run, dep)
@@ -65,7 +65,7 @@ def test_single_matrix_100_steps():
     h = 0.05
     X0, P0, G = workloads.single_matrix_inputs(256, 512, seed=0, steps=100)
     shapes = [(256, 512)]
-    run = GpuRun(shapes, hp, False, [X0], [P0])
+    run = DeviceRun(shapes, hp, False, [X0], [P0])
     ref = Tracked(shapes, [X0], [P0], depths=_depths(shapes))
     for k in range(100):
         run.set_grads([G[k]])
@@ -107,7 +107,7 @@ def test_strongly_convex_quadratic(gamma, quadratic_oracle):
     with the oracle."""
     prob = workloads.QuadraticProblem(QUAD["m"], QUAD["n"], QUAD["seed"])
     hp = HParams(QUAD["alpha"], QUAD["mu"], gamma, QUAD["eps"])
-    run = GpuRun([(QUAD["m"], QUAD["n"])], hp, False, [prob.X0], [prob.P0])
+    run = DeviceRun([(QUAD["m"], QUAD["n"])], hp, False, [prob.X0], [prob.P0])
     A = torch.from_numpy(prob.A).cuda()
     Xs = torch.from_numpy(prob.Xstar).cuda()
     A64, Xs64 = A.double(), Xs.double()
@@ -174,7 +174,7 @@ def test_edge_shapes(grad_bf16, eps, gamma):
     hp = HParams(alpha=0.3, mu=0.05, gamma=gamma, eps_stab=eps)
     X = [rng.standard_normal(workloads.array_shape(s)).astype(np.float32) for s in shapes]
     P = [(0.1 * rng.standard_normal(workloads.array_shape(s))).astype(np.float32) for s in shapes]
-    run = GpuRun(shapes, hp, grad_bf16, X, P)
+    run = DeviceRun(shapes, hp, grad_bf16, X, P)
     if eps > 0:
         for t, (m, n) in enumerate(shapes):
             R = rng.uniform(0.0, 2.0, m).astype(np.float32)
@@ -224,7 +224,7 @@ def test_degenerate_hyperparameters(case):
     shapes = EDGE_SHAPES
     X = [rng.standard_normal(workloads.array_shape(s)).astype(np.float32) for s in shapes]
     P = [(0.1 * rng.standard_normal(workloads.array_shape(s))).astype(np.float32) for s in shapes]
-    run = GpuRun(shapes, hp, True, X, P)
+    run = DeviceRun(shapes, hp, True, X, P)
     ref = Tracked.from_gpu(run, _depths(shapes))
     for k in range(3):
         g = [workloads.bf16_round(gscale * rng.standard_normal(workloads.array_shape(s)).astype(np.float32))

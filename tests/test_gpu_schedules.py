@@ -13,7 +13,7 @@ from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import workloads
 
-from gpu_helpers import GpuRun, Tracked, compare
+from gpu_helpers import DeviceRun, Tracked, compare
 
 pytestmark = pytest.mark.gpu
 
@@ -31,7 +31,7 @@ def _make(schedule, inp):
     old = os.environ.get("RIKFAD_SCHEDULE")
     os.environ["RIKFAD_SCHEDULE"] = schedule
     try:
-        return GpuRun(SHAPES, HP, True, inp.X, inp.P)
+        return DeviceRun(SHAPES, HP, True, inp.X, inp.P)
     finally:
         if old is None:
             del os.environ["RIKFAD_SCHEDULE"]
