@@ -174,7 +174,7 @@ struct rikfad_handle_s {
     // full iKFAD with shadow R-iKFAD factors (friction diagnostics)
     bool shadow = false;
     float *d_diag_u = nullptr, *d_diag_v = nullptr, *d_diag_w = nullptr, *d_diag_wpart = nullptr;
-    double *d_diag_norms = nullptr, *d_diag_upart = nullptr;
+    double *d_diag_norms = nullptr, *d_diag_upart = nullptr, *d_diag_wsq = nullptr;
     DiagState *d_diag_state = nullptr;
     DiagState *h_diag_state = nullptr;   // pinned
 
@@ -309,7 +309,7 @@ void release(rikfad_handle h)
                     (void *)h->d_slot_off, (void *)h->d_fin, (void *)h->d_fac, (void *)h->d_rowpart,
                     (void *)h->d_colpart, (void *)h->d_spart, (void *)h->d_den, (void *)h->d_guard,
                     (void *)h->d_checks, (void *)h->d_diag_u, (void *)h->d_diag_v, (void *)h->d_diag_w,
-                    (void *)h->d_diag_wpart, (void *)h->d_diag_norms, (void *)h->d_diag_upart,
+                    (void *)h->d_diag_wpart, (void *)h->d_diag_norms, (void *)h->d_diag_upart, (void *)h->d_diag_wsq,
                     (void *)h->d_diag_state, (void *)h->d_units, (void *)h->d_nodes,
                     (void *)h->d_trees, (void *)h->d_partials, (void *)h->d_counts, (void *)h->d_fetch})
         rk_free(p);
@@ -707,6 +707,7 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
         if (!rc) rc = alloc_zero(&h->d_diag_wpart, max_parts * max_n, ws);
         if (!rc) rc = alloc_zero((float **)&h->d_diag_norms, 4 * ((max_m + kWarps - 1) / kWarps), ws);
         if (!rc) rc = alloc_zero((float **)&h->d_diag_upart, 2 * ((max_m + kWarps - 1) / kWarps), ws);
+        if (!rc) rc = alloc_zero((float **)&h->d_diag_wsq, 2 * ((max_n + 31) / 32), ws);
         if (!rc) rc = alloc_zero((float **)&h->d_diag_state, (int64_t)(sizeof(DiagState) / sizeof(float)), ws);
         if (!rc) {
             cudaError_t e = rk_malloc_host((void **)&h->h_diag_state, sizeof(DiagState), cudaHostAllocDefault);
@@ -1189,12 +1190,13 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
     RK_CUDA(cudaGetLastError(), "launch diagnostic set-up kernels");
     // sigma_1 by power iteration on xi^T xi, starting from C (the shadow
     // column factor, close to the top right singular vector).  A batch of
-    // kBatch iterations (three kernels each) and the read-back of the state
+    // kBatch iterations (four kernels each) and the read-back of the state
     // record are captured once into a CUDA graph, which is replayed until
     // the iteration is done; after convergence the remaining kernels of a
-    // batch return at once.  One graph launch replaces 24 kernel launches.
+    // batch return at once.  One graph launch replaces 32 kernel launches.
     const int nb_t = (int)((m + diag_rows_per_group(m) - 1) / diag_rows_per_group(m));
     const dim3 grid_t((unsigned)nb_t, (unsigned)((n + kThreads - 1) / kThreads));
+    const int nb_c = (int)((n + 31) / 32);
     constexpr int kBatch = 8;
     DiagState &st = *h->h_diag_state;
     cudaStream_t cs = nullptr;
@@ -1217,8 +1219,10 @@ RIKFAD_API int rikfad_friction_diagnostics(rikfad_handle h, int t, int max_iters
                                                                     h->d_diag_upart, h->d_diag_state);
             rikfad_diag_matvec_t_kernel<<<grid_t, kThreads, 0, cs>>>(xi, m, n, h->d_diag_u, h->d_diag_wpart,
                                                                      h->d_diag_state);
-            rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, cs>>>(h->d_diag_wpart, nb_t, n, h->d_diag_upart,
-                                                                     nb_rows, h->d_diag_w, h->d_diag_v,
+            rikfad_diag_colsum_kernel<<<nb_c, kDiagFinThreads, 0, cs>>>(h->d_diag_wpart, nb_t, n, h->d_diag_w,
+                                                                 h->d_diag_wsq, h->d_diag_state);
+            rikfad_diag_iterate_kernel<<<1, kDiagFinThreads, 0, cs>>>(h->d_diag_w, n, h->d_diag_wsq, nb_c,
+                                                                     h->d_diag_upart, nb_rows, h->d_diag_v,
                                                                      h->d_diag_state, tol, max_iters);
         }
         cudaMemcpyAsync(h->h_diag_state, h->d_diag_state, sizeof(DiagState), cudaMemcpyDeviceToHost, cs);

@@ -6,11 +6,14 @@
 // sigma_1^2 (the comparison of the paper's Section 4.4).  sigma_1 comes from
 // power iteration on xi^T xi: two matrix-vector passes over xi per iteration
 // (HBM-bound GEMVs; there is no dense contraction to put on tensor cores).
-// The iteration runs on the device: a one-block kernel normalises the
-// iterate, forms the Rayleigh quotient and tests convergence, and every
-// kernel of the loop returns at once after convergence, so the host enqueues
-// iterations in batches and reads one small state record per batch.  Every
-// reduction runs in a fixed order.
+// The iteration runs on the device: the transposed product writes one
+// partial per row group and column, a column kernel adds them, a one-block
+// kernel normalises the iterate, forms the Rayleigh quotient and tests
+// convergence, and every kernel of the loop returns at once after
+// convergence, so the host enqueues iterations in batches and reads one small
+// state record per batch.  Every reduction runs in a fixed order.  Float64
+// is slow on this GPU: per element the kernels compute in float32, and
+// float64 only adds partial sums (per row, per column block, per block).
 #pragma once
 #include "rikfad_kernels.cuh"
 
@@ -18,11 +21,10 @@ namespace rikfad {
 
 constexpr int kDiagFinThreads = 1024;    // threads of the one-block kernels
 constexpr int kDiagBatch = 8;            // loads a thread issues before consuming them
-constexpr int kDiagMaxRowGroups = 64;    // row groups of the transposed product (partials per column)
+constexpr int kDiagMaxRowGroups = 512;   // row groups of the transposed product (partials per column)
 
-// Rows per block of the transposed product: at least 32, and few enough
-// row groups (at most kDiagMaxRowGroups) that the one-block finish sums
-// a short list of partials per column.
+// Rows per block of the transposed product: at least 32, with at most
+// kDiagMaxRowGroups row groups (partials per column for the column kernel).
 inline __host__ __device__ int64_t diag_rows_per_group(int64_t m)
 {
     const int64_t r = (m + kDiagMaxRowGroups - 1) / kDiagMaxRowGroups;
@@ -102,8 +104,11 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_setup_kernel(cons
     }
 }
 
-// Per block of 8 rows (one per warp): sum of xi^2 and of (xi - xi~)^2 in
-// float64, written to part[2 * block] and part[2 * block + 1].
+// Per block of 8 rows (one per warp): sum of xi^2 and of (xi - xi~)^2,
+// written to part[2 * block] and part[2 * block + 1].  A row is added in
+// float32 (xi - xi~ is the difference of two floats, exact where they are
+// within a factor two of each other): each lane its elements, then the 32
+// lanes by a butterfly; the rows and the blocks are added in float64.
 __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float *xi, int64_t m, int64_t n,
                                                                      const float *R, const float *C,
                                                                      const DiagState *st, double *part)
@@ -112,7 +117,7 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t row = (int64_t)blockIdx.x * kWarps + warp;
     const float inv = st->inv;
-    double a1 = 0.0, a2 = 0.0;
+    float f1 = 0.f, f2 = 0.f;
     if (row < m) {
         const float rhat = R[row] * inv;
         // kDiagBatch loads in flight per lane, then the sums in element order
@@ -126,14 +131,14 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_norms_kernel(const float
             }
 #pragma unroll
             for (int k = 0; k < kDiagBatch; ++k) {
-                const double d = (double)xv[k] - (double)(rhat * cv[k]);
-                a1 += (double)xv[k] * (double)xv[k];
-                a2 += d * d;
+                const float d = xv[k] - rhat * cv[k];
+                f1 = fmaf(xv[k], xv[k], f1);
+                f2 = fmaf(d, d, f2);
             }
         }
     }
-    a1 = warp_sum_f64(a1);
-    a2 = warp_sum_f64(a2);
+    const double a1 = (double)warp_sum(f1);
+    const double a2 = (double)warp_sum(f2);
     if (lane == 0) {
         s1[warp] = a1;
         s2[warp] = a2;
@@ -221,14 +226,57 @@ __global__ void __launch_bounds__(kThreads) rikfad_diag_matvec_t_kernel(const fl
     wpart[(int64_t)blockIdx.x * n + j] = acc;
 }
 
-// End of one power iteration, one block: w_j = sum over blocks of
-// wpart[b][j] (blocks in order), sigma^2 = ||u||^2 (the Rayleigh quotient
-// of xi^T xi at the unit v), the next iterate v = w / ||w||, and the
+// w_j = sum over the row groups of wpart[g][j] for the 32 columns of block
+// blockIdx.x (kDiagFinThreads threads): warp k adds groups k, k + 32,
+// k + 64, ... in order, then warp 0 adds the 32 warp sums in warp order.  w
+// goes to w, and the block's sum of w_j^2 (float64) to wsq[blockIdx.x].
+// Returns at once once the iteration is done.
+__global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_colsum_kernel(const float *wpart, int nb,
+                                                                             int64_t n, float *w, double *wsq,
+                                                                             const DiagState *st)
+{
+    constexpr int kColWarps = kDiagFinThreads / 32;
+    __shared__ float part[kColWarps][32];
+    if (st->done)
+        return;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t j = (int64_t)blockIdx.x * 32 + lane;
+    float acc = 0.f;
+    if (j < n) {
+        for (int g0 = warp; g0 < nb; g0 += kColWarps * kDiagBatch) {
+            float t[kDiagBatch];
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k) {
+                const int g = g0 + k * kColWarps;
+                t[k] = g < nb ? wpart[(int64_t)g * n + j] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < kDiagBatch; ++k)
+                acc += t[k];
+        }
+    }
+    part[warp][lane] = acc;
+    __syncthreads();
+    if (warp == 0) {
+        float sum = 0.f;
+#pragma unroll 8
+        for (int k = 0; k < kColWarps; ++k)
+            sum += part[k][lane];
+        if (j < n)
+            w[j] = sum;
+        const double q = warp_sum_f64(j < n ? (double)sum * (double)sum : 0.0);
+        if (lane == 0)
+            wsq[blockIdx.x] = q;
+    }
+}
+
+// End of one power iteration, one block: ||w||^2 from the column blocks'
+// partials, sigma^2 = ||u||^2 (the Rayleigh quotient of xi^T xi at the unit
+// v) from the row blocks' partials, the next iterate v = w / ||w||, and the
 // convergence test |sigma^2 - previous| <= tol sigma^2 (from the second
-// iteration on); done after max_iters iterations or when w = 0.  w is kept
-// in w_scratch between the two passes over the columns.
+// iteration on); done after max_iters iterations or when w = 0.
 __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
-    const float *wpart, int nb, int64_t n, const double *upart, int nbu, float *w_scratch, float *v,
+    const float *w, int64_t n, const double *wsq, int nbw, const double *upart, int nbu, float *v,
     DiagState *st, double tol, int max_iters)
 {
     __shared__ double scratch[kDiagFinThreads / 32 + 1];
@@ -236,20 +284,8 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
     if (st->done)
         return;
     double a = 0.0;
-    for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads) {
-        float acc = 0.f;
-        for (int b0 = 0; b0 < nb; b0 += kDiagBatch) {
-            float t[kDiagBatch];
-#pragma unroll
-            for (int k = 0; k < kDiagBatch; ++k)
-                t[k] = b0 + k < nb ? wpart[(int64_t)(b0 + k) * n + j] : 0.f;
-#pragma unroll
-            for (int k = 0; k < kDiagBatch; ++k)
-                acc += t[k];
-        }
-        w_scratch[j] = acc;
-        a += (double)acc * (double)acc;
-    }
+    for (int b = threadIdx.x; b < nbw; b += kDiagFinThreads)
+        a += wsq[b];
     const double w2 = block_sum_f64<kDiagFinThreads>(a, scratch);
     double c = 0.0;
     for (int b = threadIdx.x; b < nbu; b += kDiagFinThreads)
@@ -259,9 +295,12 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
         s_scale = w2 > 0.0 ? 1.0 / sqrt(w2) : 0.0;
     __syncthreads();
     if (w2 > 0.0) {
+        // The product in float64: rounded once, the iterate reaches a fixed
+        // point (and the quotient stops changing) instead of cycling between
+        // neighbouring float32 vectors.
         const double sc = s_scale;
         for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
-            v[j] = (float)((double)w_scratch[j] * sc);
+            v[j] = (float)((double)w[j] * sc);
     }
     if (threadIdx.x == 0) {
         const double prev = st->sigma2;
