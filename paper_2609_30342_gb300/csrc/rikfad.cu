@@ -998,6 +998,7 @@ RIKFAD_API int rikfad_enqueue_denominators(rikfad_handle h, float *host_out, voi
     if (T == 0)
         return RIKFAD_OK;
     cudaStream_t s = (cudaStream_t)stream;
+    RK_CUDA(cudaPeekAtLastError(), "earlier CUDA error");
     // Page-locked memory mapped into the device's address space takes the
     // kernel's stores directly, so no copy sits between this step's finalise
     // and the next step's kernels (PDL launches chain through); other host
