@@ -159,7 +159,10 @@ RIKFAD_API void rikfad_destroy(rikfad_handle h);
  * call (a change costs one small host-to-device copy).  Every pointer must be
  * 16-byte aligned, except for matrices whose cols is not a multiple of 8 and
  * for which only natural alignment is required.  Pointers of empty tensors
- * may be NULL.  x, grad and p must not overlap.
+ * may be NULL.  x, grad and p must not overlap.  When a pointer differs from
+ * the previous call's, the host checks that the device can address it
+ * (RIKFAD_ERR_ARG for memory of another device, or for pageable host memory
+ * on a device that cannot read it through the host's page tables).
  *
  * Stored form of the momentum of a matrix: between steps p holds P^(1) of
  * the last step (the half-damped momentum) and the library remembers the

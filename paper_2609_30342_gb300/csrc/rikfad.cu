@@ -141,6 +141,7 @@ int report_error(int code, const std::string &msg)
 
 struct rikfad_handle_s {
     int device = 0;
+    bool pageable_ok = false;       // the device reads pageable host memory (host page tables)
     int ntensors = 0;
     int grad_bytes = 4;
     rikfad_hparams hp{};
@@ -264,6 +265,36 @@ void ptrtable_free(PtrTable &t)
     if (t.uploaded)
         cudaEventDestroy(t.uploaded);
     t = PtrTable();
+}
+
+// Every pointer the kernels will dereference must be memory this device can
+// address: its own device memory, page-locked host memory, or pageable host
+// memory when the device reads that through the host's page tables
+// (pageable_ok).  Checked on the host for the entries that changed, so a
+// wrong pointer is an argument error instead of a device fault.  `what`
+// names the list entries: entry i is tensor i % ntensors of list i / ntensors.
+int check_pointers(const PtrTable &t, const std::vector<void *> &want, int device, bool pageable_ok,
+                   int ntensors, const char *const *lists)
+{
+    for (int i = 0; i < t.count; ++i) {
+        if (want[i] == nullptr || (t.valid && want[i] == t.cached[i]))
+            continue;
+        cudaPointerAttributes a{};
+        const cudaError_t e = cudaPointerGetAttributes(&a, want[i]);
+        const std::string where = std::string(lists[i / ntensors]) + " pointer of tensor " +
+                                  std::to_string(i % ntensors);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(RIKFAD_ERR_ARG, where + " is not an address CUDA recognises");
+        }
+        if (a.type == cudaMemoryTypeDevice && a.device != device)
+            return fail(RIKFAD_ERR_ARG, where + " is memory of device " + std::to_string(a.device) +
+                                            ", not of the handle's device " + std::to_string(device));
+        if (a.type == cudaMemoryTypeUnregistered && !pageable_ok)
+            return fail(RIKFAD_ERR_ARG, where + " is pageable host memory, which this device cannot "
+                                                "read; use device or page-locked host memory");
+    }
+    return RIKFAD_OK;
 }
 
 // Make the device table equal `want`; enqueue the copy on `stream` if needed.
@@ -463,7 +494,11 @@ int canonical(rikfad_handle h, const float *const *src, float *const *dst, bool 
         want[T + t] = (void *)dst[t];
     }
     if (h->plan.nblocks > 0) {
-        int rc = ptrtable_set(h->canon_ptrs, want, stream);
+        static const char *const lists[2] = {"source momentum", "destination momentum"};
+        int rc = check_pointers(h->canon_ptrs, want, h->device, h->pageable_ok, T, lists);
+        if (rc)
+            return rc;
+        rc = ptrtable_set(h->canon_ptrs, want, stream);
         if (rc)
             return rc;
         CanonParams c{};
@@ -599,6 +634,8 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
     int dev = 0, sms = 0, occ = 0;
     RK_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
     RK_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+    int pageable = 0;
+    RK_CUDA(cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev), "cudaDeviceGetAttribute");
     // Persistent grid: as many blocks as can be resident at once.
     int occ_min = 1 << 30;
     const void *kernels[6] = {(const void *)rikfad_step_kernel<float, true>,
@@ -636,6 +673,7 @@ int create_impl(const rikfad_shape *shapes, int ntensors, const rikfad_hparams *
 
     rikfad_handle h = new rikfad_handle_s();
     h->device = dev;
+    h->pageable_ok = pageable != 0;
     h->ntensors = ntensors;
     h->grad_bytes = grad_dtype == RIKFAD_GRAD_BF16 ? 2 : 4;
     h->hp = *hp;
@@ -794,6 +832,10 @@ RIKFAD_API int rikfad_step(rikfad_handle h, double step, float *const *x, const 
     cudaStream_t s = (cudaStream_t)stream;
     RK_CUDA(cudaPeekAtLastError(), "earlier CUDA error");
     if (h->plan.nblocks > 0) {
+        static const char *const lists[3] = {"x", "grad", "p"};
+        rc = check_pointers(h->step_ptrs, want, h->device, h->pageable_ok, T, lists);
+        if (rc)
+            return rc;
         rc = ptrtable_set(h->step_ptrs, want, s);
         if (rc)
             return rc;

@@ -305,3 +305,30 @@ def test_enqueued_denominators_match_the_synchronous_read():
     torch.cuda.synchronize()
     assert np.array_equal(pageable, expect[-1])
     run.close()
+
+
+def test_host_pointers_are_checked_before_any_launch():
+    """A changed pointer is checked on the host: pageable host memory for a
+    gradient either works in place (a device that reads pageable memory
+    through the host's page tables, as GB300 does) and gives bitwise the
+    step of a device copy, or is refused with RIKFAD_ERR_ARG before any
+    kernel runs; the handle stays usable either way."""
+    inp, run_d = _run()
+    _, run_h = _run()
+    g = inp.grads(0)
+    run_d.set_grads(g)
+    run_h.set_grads(g)
+    pageable = [np.ascontiguousarray(torch.from_numpy(a).to(torch.bfloat16).view(torch.int16).numpy())
+                for a in g]
+    ptrs = [a.ctypes.data for a in pageable]
+    try:
+        run_h.opt.step(0.1, run_h.x, ptrs, run_h.p)
+    except rikfad.RikfadError as e:
+        assert e.code == rikfad.ERR_ARG and "pageable host memory" in str(e)
+        run_h.step(0.1)                      # the device gradients still step
+    run_d.step(0.1)
+    torch.cuda.synchronize()
+    for a, b in zip(run_d.x + run_d.p, run_h.x + run_h.p):
+        assert torch.equal(a, b)
+    run_d.close()
+    run_h.close()
