@@ -70,6 +70,7 @@ __device__ __forceinline__ bool fin_item_ok(const FinParams &f, const FinItemDev
         return true;
     const PanelDev pd = f.panels[it.panel];
     const int ns = pd.slot_end - pd.slot_begin;
+    (void)ns;                  // read by the checks only
     return RK_DEV_CHECK(cb, pd.tensor == it.tensor && pd.col0 >= 0 &&
                                 (int64_t)pd.col0 + pd.width <= td.cols, kChkCols) &&
            RK_DEV_CHECK(cb, it.begin >= 0 && it.begin <= it.end && it.end <= pd.width, kChkCols) &&
