@@ -33,6 +33,9 @@
  *     are detected before any work is enqueued.  Errors of work already
  *     enqueued surface as RIKFAD_ERR_CUDA on a later call.
  *   - A handle is not thread-safe: calls on one handle must not overlap.
+ *     Its device work shares the handle's workspace and state, so it must
+ *     also be ordered on the GPU: enqueue it on one stream, or order the
+ *     streams with events.
  *   - Non-finite guard.  The friction of Eq. xi_def divides by 1^T R +
  *     eps_stab and every element of a matrix reads R and C, so one
  *     non-finite gradient or momentum element poisons its whole matrix
