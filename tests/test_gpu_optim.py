@@ -1,0 +1,61 @@
+"""The torch.optim front end (paper_2609_30342_gb300.optim): a small model
+trained a few steps with RIKFADOptimizer takes bitwise the steps of the
+pointer API on the same gradients (a parameter without a gradient steps with
+a zero gradient), and its materialised momenta equal the pointer API's."""
+import pytest
+import torch
+
+from paper_2609_30342_gb300 import build as pkg_build
+from paper_2609_30342_gb300 import rikfad
+from paper_2609_30342_gb300.optim import RIKFADOptimizer
+
+pytestmark = pytest.mark.gpu
+
+HP = dict(alpha=0.2, mu=1e-3, gamma=0.05, eps_stab=1e-8)
+H = 0.05
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    pkg_build.build()
+    yield
+
+
+def test_optimizer_matches_the_pointer_api():
+    torch.manual_seed(0)
+    model = torch.nn.Sequential(torch.nn.Linear(64, 96), torch.nn.GELU(), torch.nn.LayerNorm(96),
+                                torch.nn.Linear(96, 10)).cuda()
+    params = list(model.parameters())
+    ref = [p.detach().clone() for p in params]
+    mom = [torch.zeros_like(p) for p in params]
+    shapes = [(p.shape[0], p.shape[1]) if p.dim() == 2 else (p.numel(), 0) for p in params]
+    api = rikfad.RIKFAD(shapes, grad_dtype="f32", **HP)
+    opt = RIKFADOptimizer(params, lr=H, **HP)
+    x = torch.randn(32, 64, device="cuda")
+    y = torch.randint(0, 10, (32,), device="cuda")
+    for k in range(4):
+        opt.zero_grad()
+        torch.nn.functional.cross_entropy(model(x), y).backward()
+        if k == 2:
+            params[1].grad = None             # no gradient this step: a zero gradient
+        grads = [torch.zeros_like(p) if p.grad is None else p.grad.detach().clone() for p in params]
+        opt.step()
+        api.step(H, ref, grads, mom)
+        torch.cuda.synchronize()
+        for a, b in zip(params, ref):
+            assert torch.equal(a.detach(), b)
+    opt.materialize()
+    api.materialize(mom)
+    torch.cuda.synchronize()
+    for p, m in zip(params, mom):
+        assert torch.equal(opt.state[p]["momentum"], m)
+    opt.check_finite()
+    opt.close()
+    api.close()
+
+
+def test_optimizer_rejects_cpu_parameters():
+    opt = RIKFADOptimizer([torch.nn.Parameter(torch.zeros(4, 4))], lr=H, **HP)
+    opt.param_groups[0]["params"][0].grad = torch.zeros(4, 4)
+    with pytest.raises(ValueError):
+        opt.step()
