@@ -6,6 +6,8 @@ friction rule, every other shape element-wise (Section 2 of the paper; ``lr`` is
 the step size h).  It is argument marshalling only: a group's handle is created
 at its first step, the momentum buffers live in ``self.state[p]["momentum"]`` in
 the library's stored form, and ``materialize()`` turns them into the paper's P.
+``state_dict()`` also carries each group's library state image, so a checkpoint
+resumes the exact trajectory.
 Parameters and their gradients must be contiguous float32 CUDA tensors of one
 device (autograd gives a float32 parameter a float32 gradient; bfloat16
 gradients are for the pointer API, ``rikfad.RIKFAD``).  A parameter without a
@@ -22,15 +24,15 @@ class RIKFADOptimizer(torch.optim.Optimizer):
             raise ValueError("lr (the step size h) must be > 0")
         defaults = dict(lr=lr, alpha=alpha, mu=mu, gamma=gamma, eps_stab=eps_stab)
         super().__init__(params, defaults)
-        self._groups = {}     # id(group) -> (handle, parameter list, zero gradients)
+        self._groups = {}     # group index -> (handle, parameter list, zero gradients)
 
     @staticmethod
     def _shape(p):
         return (p.shape[0], p.shape[1]) if p.dim() == 2 else (p.numel(), 0)
 
-    def _group_handle(self, group):
+    def _group_handle(self, i, group):
         params = group["params"]
-        entry = self._groups.get(id(group))
+        entry = self._groups.get(i)
         if entry is not None and len(entry[1]) == len(params) and all(a is b for a, b in zip(entry[1], params)):
             return entry
         if entry is not None:
@@ -43,7 +45,7 @@ class RIKFADOptimizer(torch.optim.Optimizer):
         handle = rikfad.RIKFAD([self._shape(p) for p in params], group["alpha"], group["mu"],
                                group["gamma"], group["eps_stab"], grad_dtype="f32")
         entry = (handle, list(params), [torch.zeros_like(p) for p in params])
-        self._groups[id(group)] = entry
+        self._groups[i] = entry
         return entry
 
     def _momenta(self, params):
@@ -61,10 +63,10 @@ class RIKFADOptimizer(torch.optim.Optimizer):
         if closure is not None:
             with torch.enable_grad():
                 loss = closure()
-        for group in self.param_groups:
+        for i, group in enumerate(self.param_groups):
             if not group["params"]:
                 continue
-            handle, params, zeros = self._group_handle(group)
+            handle, params, zeros = self._group_handle(i, group)
             grads = []
             for p, z in zip(params, zeros):
                 g = p.grad
@@ -80,6 +82,33 @@ class RIKFADOptimizer(torch.optim.Optimizer):
         """Turn every momentum buffer into the paper's P_{n+1} (in place)."""
         for handle, params, _ in self._groups.values():
             handle.materialize(self._momenta(params), stream=torch.cuda.current_stream(params[0].device))
+
+    def state_dict(self):
+        """torch's state (the momentum buffers, in the stored form) plus each
+        group's library state image (factors, element-wise friction and the
+        pending step size; rikfad_export_state) as a CPU byte tensor."""
+        sd = super().state_dict()
+        images = {}
+        for i, group in enumerate(self.param_groups):
+            entry = self._groups.get(i)
+            if entry is not None:
+                handle, params, _ = entry
+                img = torch.empty(handle.state_image_bytes(), dtype=torch.uint8, device=params[0].device)
+                handle.export_state(img, stream=torch.cuda.current_stream(params[0].device))
+                images[i] = img.cpu()
+        sd["rikfad_images"] = images
+        return sd
+
+    def load_state_dict(self, state_dict):
+        sd = dict(state_dict)
+        images = sd.pop("rikfad_images", {})
+        self.close()          # the groups are replaced; handles are made again below or at the next step
+        super().load_state_dict(sd)
+        for i, group in enumerate(self.param_groups):
+            if i in images:
+                handle, params, _ = self._group_handle(i, group)
+                img = images[i].to(params[0].device)
+                handle.import_state(img, stream=torch.cuda.current_stream(params[0].device))
 
     def check_finite(self):
         """Raise rikfad.RikfadError(ERR_NONFINITE) if a step produced a

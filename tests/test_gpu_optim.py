@@ -2,6 +2,8 @@
 trained a few steps with RIKFADOptimizer takes bitwise the steps of the
 pointer API on the same gradients (a parameter without a gradient steps with
 a zero gradient), and its materialised momenta equal the pointer API's."""
+import io
+
 import pytest
 import torch
 
@@ -59,3 +61,40 @@ def test_optimizer_rejects_cpu_parameters():
     opt.param_groups[0]["params"][0].grad = torch.zeros(4, 4)
     with pytest.raises(ValueError):
         opt.step()
+
+
+def test_state_dict_resumes_the_trajectory():
+    """A checkpoint of the model and the optimiser (torch state plus the
+    library's state image) taken after two steps and written with torch.save,
+    loaded into a fresh optimiser over a fresh model, gives bitwise the same
+    third step."""
+    torch.manual_seed(1)
+    model = torch.nn.Sequential(torch.nn.Linear(48, 80), torch.nn.Tanh(), torch.nn.Linear(80, 8)).cuda()
+    opt = RIKFADOptimizer(model.parameters(), lr=H, **HP)
+    x = torch.randn(16, 48, device="cuda")
+    y = torch.randn(16, 8, device="cuda")
+
+    def loss(m):
+        return torch.nn.functional.mse_loss(m(x), y)
+
+    for _ in range(2):
+        opt.zero_grad()
+        loss(model).backward()
+        opt.step()
+    buf = io.BytesIO()                     # a checkpoint: serialised, so nothing is shared
+    torch.save({"model": model.state_dict(), "opt": opt.state_dict()}, buf)
+    buf.seek(0)
+    ckpt = torch.load(buf)
+    clone = torch.nn.Sequential(torch.nn.Linear(48, 80), torch.nn.Tanh(), torch.nn.Linear(80, 8)).cuda()
+    clone.load_state_dict(ckpt["model"])
+    opt2 = RIKFADOptimizer(clone.parameters(), lr=H, **HP)
+    opt2.load_state_dict(ckpt["opt"])
+    for m, o in ((model, opt), (clone, opt2)):
+        o.zero_grad()
+        loss(m).backward()
+        o.step()
+    torch.cuda.synchronize()
+    for a, b in zip(model.parameters(), clone.parameters()):
+        assert torch.equal(a.detach(), b.detach())
+    opt.close()
+    opt2.close()
