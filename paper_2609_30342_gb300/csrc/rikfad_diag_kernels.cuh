@@ -295,9 +295,8 @@ __global__ void __launch_bounds__(kDiagFinThreads) rikfad_diag_iterate_kernel(
         s_scale = w2 > 0.0 ? 1.0 / sqrt(w2) : 0.0;
     __syncthreads();
     if (w2 > 0.0) {
-        // The product in float64: rounded once, the iterate reaches a fixed
-        // point (and the quotient stops changing) instead of cycling between
-        // neighbouring float32 vectors.
+        // The product in float64, rounded once (scaled in float32 the quotient
+        // seldom settled to a 1e-10 convergence test).
         const double sc = s_scale;
         for (int64_t j = threadIdx.x; j < n; j += kDiagFinThreads)
             v[j] = (float)((double)w[j] * sc);
