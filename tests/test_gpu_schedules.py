@@ -8,7 +8,6 @@ import numpy as np
 import pytest
 import torch
 
-import oracle
 from oracle import HParams
 from paper_2609_30342_gb300 import build as pkg_build
 from paper_2609_30342_gb300 import workloads
