@@ -4,7 +4,8 @@ offset and each pointer-table entry before using it, counting failures
 instead of trapping.  The edge-shape, degenerate-hyperparameter,
 Nano-shaped and full GPT2-S (the benchmark's launch configuration) parity
 cases, the C-ABI behaviour tests, full iKFAD, the shadow
-handle and the in-order schedule run on it in a child process (the library
+handle, the in-order schedule and the torch.optim front end run on it in a
+child process (the library
 is chosen when the binding first loads it), and every handle must end with
 zero failed checks; the parity assertions themselves hold as on the
 ordinary build."""
@@ -30,7 +31,7 @@ def test_parity_cases_on_checked_build():
                  "gpt2_small_full_size",
            os.path.join(HERE, "test_gpu_parity.py"), os.path.join(HERE, "test_gpu_api.py"),
            os.path.join(HERE, "test_gpu_ikfad.py"), os.path.join(HERE, "test_gpu_diagnostics.py"),
-           os.path.join(HERE, "test_gpu_schedules.py")]
+           os.path.join(HERE, "test_gpu_schedules.py"), os.path.join(HERE, "test_gpu_optim.py")]
     r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=1500)
     tail = (r.stdout + r.stderr)[-3000:]
     assert r.returncode == 0, tail

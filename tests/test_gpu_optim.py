@@ -3,6 +3,7 @@ trained a few steps with RIKFADOptimizer takes bitwise the steps of the
 pointer API on the same gradients (a parameter without a gradient steps with
 a zero gradient), and its materialised momenta equal the pointer API's."""
 import io
+import os
 
 import pytest
 import torch
@@ -21,6 +22,19 @@ H = 0.05
 def built():
     pkg_build.build()
     yield
+
+
+def _no_failed_checks(*handles):
+    """On the checked build (its child run sets RIKFAD_EXPECT_CHECKED), no
+    device-side plan check may have failed."""
+    if os.environ.get("RIKFAD_EXPECT_CHECKED"):
+        for h in handles:
+            n, code = h.debug_check_failures()
+            assert n == 0, "device-side plan checks failed: %d (first code %d)" % (n, code)
+
+
+def _handles(opt):
+    return [entry[0] for entry in opt._groups.values()]
 
 
 def test_optimizer_matches_the_pointer_api():
@@ -52,6 +66,7 @@ def test_optimizer_matches_the_pointer_api():
     for p, m in zip(params, mom):
         assert torch.equal(opt.state[p]["momentum"], m)
     opt.check_finite()
+    _no_failed_checks(api, *_handles(opt))
     opt.close()
     api.close()
 
@@ -96,5 +111,6 @@ def test_state_dict_resumes_the_trajectory():
     torch.cuda.synchronize()
     for a, b in zip(model.parameters(), clone.parameters()):
         assert torch.equal(a.detach(), b.detach())
+    _no_failed_checks(*_handles(opt), *_handles(opt2))
     opt.close()
     opt2.close()
