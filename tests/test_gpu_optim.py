@@ -71,12 +71,6 @@ def test_optimizer_matches_the_pointer_api():
     api.close()
 
 
-def test_optimizer_rejects_cpu_parameters():
-    opt = RIKFADOptimizer([torch.nn.Parameter(torch.zeros(4, 4))], lr=H, **HP)
-    opt.param_groups[0]["params"][0].grad = torch.zeros(4, 4)
-    with pytest.raises(ValueError):
-        opt.step()
-
 
 def test_state_dict_resumes_the_trajectory():
     """A checkpoint of the model and the optimiser (torch state plus the
